@@ -1,0 +1,439 @@
+#!/usr/bin/env python
+"""Tree-verify benchmark: verify steps/s at the 7B shape (KV 2400, 64-node
+tree) and the HBM roofline of the attention kernel.
+
+One step = 6 draft-layer expansions (width 8) over 65536-entry draft rows,
+the top-63 rerank, tree attention over all 32 layers (32 heads x 128, prefix
+2400), the acceptance walk and the KV commit of the accepted path: every row
+of the hot path, as one sequence of library launches (three CUDA graphs).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 7b|llamagen|c1]
+                  [--mode greedy|spec_det] [--impl adt|reference]
+
+Prints one JSON line.  With torchrun (N > 1) every rank runs an independent
+replica on its own GPU (the path has no cross-GPU exchange) and rank 0
+reports the whole-job throughput (weak scaling).
+"""
+from __future__ import annotations
+
+import argparse
+import datetime as _dt
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOADS = {
+    "7b": dict(name="7B-class (Anole / Lumina-mGPT shape) tree verify: 32 layers, 32 heads x 128, KV 2400, "
+                    "64-node tree (depth 6, width 8), vocab 65536, batch 1",
+               layers=32, H=32, Hkv=32, D=128, V=65536, kv_len=[2400], depth=[6], width=[8], max_nodes=64),
+    "llamagen": dict(name="LlamaGen-XL-shaped tree verify: 36 layers, 20 heads x 64, KV 696 (120 text + 576 image), "
+                          "64-node tree (depth 6, width 8), vocab 16384, batch 1",
+                     layers=36, H=20, Hkv=20, D=64, V=16384, kv_len=[696], depth=[6], width=[8], max_nodes=64),
+    "c1": dict(name="single verify step: 1 layer, 8 heads x 64, KV 512, 26-node tree (depth 4, width 4), "
+                    "vocab 16384, batch 1",
+               layers=1, H=8, Hkv=8, D=64, V=16384, kv_len=[512], depth=[4], width=[4], max_nodes=26),
+}
+
+# DRAM bytes (read + write) of one tree_attn launch at the 7B shape, from one
+# ncu capture; valid only for the kernel source with this SHA-256 prefix.
+NCU_TRAFFIC = {}
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def attn_source_sha():
+    with open(os.path.join(ROOT, "paper_2512_21857_gb300", "csrc", "tree_attn.cu"), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, device_index):
+        self.dev = device_index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "100", "-i", str(self.dev)], stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self, t0, t1):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = []
+        for line in out.splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 10:
+                continue
+            try:
+                ts = _dt.datetime.strptime(parts[0], "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                rows.append((ts, float(parts[2]), float(parts[3]), parts[6:10]))
+            except ValueError:
+                continue
+        inside = [r for r in rows if t0 - 0.05 <= r[0] <= t1 + 0.05]
+        use = inside or rows
+        if not use:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        reasons = sorted({n for r in use for n, v in zip(self.NAMES, r[3]) if v.lower().startswith("active")})
+        return {"sm_mhz": statistics.median(r[1] for r in use), "sm_max_mhz": max(r[2] for r in use),
+                "reasons": reasons, "samples": len(use), "samples_in_timed_region": len(inside)}
+
+
+# ------------------------------------------------------------------ GPU arm
+
+def fill_inputs_on_device(step, seed):
+    """Seeded synthetic inputs drawn on the device (bf16 ~ N(0,1) caches and
+    projections, fp32 ~ N(0, 3^2) logits, 24-bit uniforms)."""
+    import torch
+    g = torch.Generator(device=step.device)
+    g.manual_seed(seed)
+
+    def normal_(t, std=1.0):
+        t.copy_((torch.randn(t.shape, generator=g, device=step.device) * std).to(t.dtype))
+
+    for name in ("k_cache", "v_cache", "q", "k_tree", "v_tree"):
+        normal_(getattr(step, name))
+    for rows in step.draft_rows:
+        normal_(rows, 3.0)
+    normal_(step.target, 3.0)
+    for t in (step.u_accept, step.u_sample):
+        t.copy_(torch.randint(0, 1 << 24, t.shape, generator=g, device=step.device).float() * 2.0 ** -24)
+    step.root_token.copy_(torch.randint(0, step.shape.V, step.root_token.shape, generator=g, device=step.device))
+
+
+def run_gpu(args, wl, rank, world):
+    import torch
+    from paper_2512_21857_gb300 import binding as B
+    from paper_2512_21857_gb300 import build as libbuild
+    from paper_2512_21857_gb300.verify_step import StepShape, TreeVerifyStep
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    libbuild.build()
+    B.lib()
+    mode = {"greedy": B.ACCEPT_GREEDY, "spec_det": B.ACCEPT_SPEC_DET}[args.mode]
+    shape = StepShape(layers=wl["layers"], H=wl["H"], Hkv=wl["Hkv"], D=wl["D"], V=wl["V"], kv_len=wl["kv_len"],
+                      depth=wl["depth"], width=wl["width"], max_nodes=wl["max_nodes"], mode=mode, temperature=1.0)
+    step = TreeVerifyStep(shape)
+    fill_inputs_on_device(step, 20251221 + rank)
+    stream = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    # eager pass first (per-device one-time set-up happens outside capture)
+    with torch.cuda.stream(stream):
+        step.launch(stream)
+    torch.cuda.synchronize()
+    if B.adt_get_device_error(stream) != 0:
+        raise RuntimeError("device error flag set during the eager pass")
+    graphs = [torch.cuda.CUDAGraph() for _ in range(3)]
+    with torch.cuda.stream(stream):
+        with torch.cuda.graph(graphs[0], stream=stream):
+            step.launch_draft(stream)
+        with torch.cuda.graph(graphs[1], stream=stream):
+            for layer in range(shape.layers):
+                step.launch_attention(layer, stream)
+        with torch.cuda.graph(graphs[2], stream=stream):
+            step.launch_verify(stream)
+    torch.cuda.synchronize()
+
+    def one_step(ev_a=None, ev_b=None):
+        graphs[0].replay()
+        if ev_a is not None:
+            ev_a.record(stream)
+        graphs[1].replay()
+        if ev_b is not None:
+            ev_b.record(stream)
+        graphs[2].replay()
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            one_step()
+    torch.cuda.synchronize()
+
+    K = args.steps
+    ev_a = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.4)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    t0 = time.time()
+    with torch.cuda.stream(stream):
+        ev0.record(stream)
+        for i in range(K):
+            one_step(ev_a[i], ev_b[i])
+        ev1.record(stream)
+    torch.cuda.synchronize()
+    t1 = time.time()
+    if world > 1:
+        torch.distributed.barrier()
+    clocks = sampler.stop(t0, t1)
+    step_ms = ev0.elapsed_time(ev1) / K
+    attn_ms = sum(a.elapsed_time(b) for a, b in zip(ev_a, ev_b)) / (K * shape.layers)
+    errbits = B.adt_get_device_error(stream)
+    if errbits:
+        raise RuntimeError(f"device error bits {errbits:#x} during the timed steps")
+    if world > 1:
+        t = torch.tensor([step_ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        step_ms = float(t.item())
+
+    # end to end through the public API: per-step inputs copied from pinned
+    # host memory, results read back, host synchronised every step
+    per_step_inputs = [step.q, step.k_tree, step.v_tree, step.target, step.u_accept, step.u_sample,
+                       step.root_token] + list(step.draft_rows)
+    host_in = [t.cpu().pin_memory() for t in per_step_inputs]
+    outputs = [step.path, step.accept_len, step.bonus, step.kv_len_out]
+    host_out = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in outputs]
+    h2d = sum(t.numel() * t.element_size() for t in host_in)
+    d2h = sum(t.numel() * t.element_size() for t in host_out)
+    K2 = max(3, min(K, args.e2e_steps))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(K2):
+            for d, h in zip(per_step_inputs, host_in):
+                d.copy_(h, non_blocking=True)
+            one_step()
+            for h, d in zip(host_out, outputs):
+                h.copy_(d, non_blocking=True)
+            stream.synchronize()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / K2
+    if world > 1:
+        t = torch.tensor([e2e_ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+
+    ab = step.algorithmic_bytes()
+    peak, peak_kind = measured_peaks()
+    achieved = ab["attention_per_layer"] / (attn_ms * 1e-3) / 1e9
+    sha = attn_source_sha()
+    traffic = NCU_TRAFFIC.get(sha) if args.workload == "7b" else None
+    return dict(step_ms=step_ms, attn_ms=attn_ms, clocks=clocks, e2e_ms=e2e_ms, h2d=h2d, d2h=d2h,
+                launches=K * step.kernel_launches_per_step(), achieved=achieved, peak=peak, peak_kind=peak_kind,
+                traffic=traffic, attn_bytes=ab["attention_per_layer"], step_bytes=ab["attention"], sha=sha)
+
+
+# ------------------------------------------------------------------ oracle (CPU) samples
+
+class OracleSample:
+    """A bounded sample of one verify step run by the oracle, extrapolated to
+    the full step: `heads` query heads of `layers_sampled` layers of
+    attention (all tree nodes), `rows_sampled` draft rows of expansion, the
+    full rerank and greedy acceptance walk, and the KV commit of one layer.
+    Inputs are drawn once; run() times only the oracle calls."""
+
+    def __init__(self, wl, seed, heads, layers_sampled, rows_sampled):
+        import numpy as np
+
+        from paper_2512_21857_gb300 import synth
+
+        self.wl = wl
+        H, Hkv, D, V, L = wl["H"], wl["Hkv"], wl["D"], wl["V"], wl["kv_len"][0]
+        k, depth, nmax = wl["width"][0], wl["depth"][0], wl["max_nodes"]
+        self.n = n = min(nmax, k + (depth - 1) * k * k + 1)
+        self.hs = hs = max(1, min(heads, H))
+        self.layers_sampled = layers_sampled
+        self.rows_sampled = rows_sampled
+        self.total_rows = 1 + (depth - 1) * k
+        g = synth.rng(seed, "oracle_sample")
+        self.tb = synth.tree_batch([n], V, seed)
+        self.q = synth.bf16_normal((n, hs, D), seed, "q").double().numpy()
+        self.kc = synth.bf16_normal((1, hs, L, D), seed, "kc").double().numpy()
+        self.vc = synth.bf16_normal((1, hs, L, D), seed, "vc").double().numpy()
+        self.kt = synth.bf16_normal((n, hs, D), seed, "kt").double().numpy()
+        self.vt = synth.bf16_normal((n, hs, D), seed, "vt").double().numpy()
+        self.rows = synth.f32_normal((rows_sampled, V), seed, "rows")
+        self.target = synth.f32_normal((n, V), seed, "target")
+        C = k + (depth - 1) * k * k
+        self.cand_tok = g.integers(0, V, size=C).astype(np.int32)
+        self.cand_score = -np.sort(g.random(C)).astype(np.float32)
+        self.cand_par = -np.ones(C, np.int32)
+        self.kc16 = np.zeros((1, 1, Hkv, L + nmax, D), np.int16)
+        self.kt16 = np.zeros((1, n, Hkv, D), np.int16)
+        self.desc = (f"oracle (numpy fp64, 1 thread) on {hs} of {H} heads x {layers_sampled} of {wl['layers']} "
+                     f"layers of attention, {rows_sampled} of {self.total_rows} draft rows of expansion, full "
+                     f"rerank and greedy walk, 1 of {wl['layers']} layers of KV commit; extrapolated linearly "
+                     f"to one full step")
+
+    def run(self):
+        import numpy as np
+
+        import oracle
+
+        wl = self.wl
+        L, D, n, k = wl["kv_len"][0], wl["D"], self.n, wl["width"][0]
+        t = time.perf_counter()
+        for _ in range(self.layers_sampled):
+            oracle.tree_attention(self.q, self.kc, self.vc, [L], self.kt, self.vt, self.tb.parents, [0, n],
+                                  1.0 / math.sqrt(D))
+        t_attn = (time.perf_counter() - t) / self.layers_sampled * wl["layers"] * (wl["H"] / self.hs)
+        t = time.perf_counter()
+        oracle.tree_expand(self.rows, np.zeros(self.rows_sampled, np.float32), k, k)
+        t_exp = (time.perf_counter() - t) / self.rows_sampled * self.total_rows
+        t = time.perf_counter()
+        oracle.tree_rerank(self.cand_tok, self.cand_score, self.cand_par, 1, n)
+        oracle.tree_accept(self.target, None, self.tb.tokens, self.tb.parents, [0, n], oracle.ACCEPT_GREEDY)
+        t_acc = time.perf_counter() - t
+        t = time.perf_counter()
+        oracle.kv_compact(self.kc16, self.kc16, [L], self.kt16, self.kt16, [0, n], [[0, 1]])
+        t_cmp = (time.perf_counter() - t) * wl["layers"]
+        return t_attn + t_exp + t_acc + t_cmp
+
+
+def cpu_sample_subprocess(wl_key, heads, layers_sampled, rows_sampled, reps):
+    """Runs oracle samples in a fresh single-threaded process."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               CUDA_VISIBLE_DEVICES="")
+    cmd = [sys.executable, os.path.abspath(__file__), "--cpu-sample", wl_key, "--cpu-heads", str(heads),
+           "--cpu-layers", str(layers_sampled), "--cpu-rows", str(rows_sampled), "--cpu-reps", str(reps)]
+    out = subprocess.run(cmd, capture_output=True, text=True, env=env, timeout=1800)
+    if out.returncode != 0:
+        raise RuntimeError(out.stderr[-2000:])
+    return json.loads(out.stdout.strip().splitlines()[-1])
+
+
+def cpu_sample_main(args):
+    wl = WORKLOADS[args.cpu_sample]
+    sample = OracleSample(wl, 7, args.cpu_heads, args.cpu_layers, args.cpu_rows)
+    times = [sample.run() for _ in range(args.cpu_reps)]
+    print(json.dumps({"sec_per_step": times, "desc": sample.desc}))
+
+
+# ------------------------------------------------------------------ main
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--workload", default="7b", choices=sorted(WORKLOADS))
+    ap.add_argument("--mode", default="greedy", choices=["greedy", "spec_det"])
+    ap.add_argument("--impl", default="adt", choices=["adt", "reference"])
+    ap.add_argument("--e2e-steps", type=int, default=200)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-sample", default=None)
+    ap.add_argument("--cpu-heads", type=int, default=1)
+    ap.add_argument("--cpu-layers", type=int, default=1)
+    ap.add_argument("--cpu-rows", type=int, default=1)
+    ap.add_argument("--cpu-reps", type=int, default=1)
+    args = ap.parse_args()
+    if args.cpu_sample:
+        cpu_sample_main(args)
+        return
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be >= 3")
+    wl = WORKLOADS[args.workload]
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    config = {"workload": wl["name"], "batch": len(wl["kv_len"]), "kv_len": wl["kv_len"][0],
+              "tree_nodes": wl["max_nodes"], "depth": wl["depth"][0], "width": wl["width"][0], "vocab": wl["V"],
+              "layers": wl["layers"], "heads": wl["H"], "head_dim": wl["D"], "accept_mode": args.mode,
+              "l2": "inputs larger than L2: every layer reads its own 39 MB KV cache slice (1.3 GB per step)"
+                    if args.workload == "7b" else "per-step inputs rotate through distinct layer buffers",
+              "parallelism": f"replicas x{world}"}
+    metric = "tree-verify steps/s"
+
+    if args.impl == "reference":
+        # The reference arm is the CPU oracle: each of the W + K steps times a
+        # bounded sample of one verify step (one head of one layer of
+        # attention, one draft row of expansion, the full rerank and walk,
+        # one layer of KV commit) and extrapolates it to the full step.
+        if rank != 0:
+            return
+        t_run = time.time()
+        res = cpu_sample_subprocess(args.workload, 1, 1, 1, args.warmup + args.steps)
+        samples = res["sec_per_step"][args.warmup:]
+        sec = statistics.mean(samples)
+        value = 1.0 / sec
+        line = {"impl": "reference", "metric": metric, "value": value, "unit": "steps/s", "n_gpus": world,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": config,
+                "cpu_baseline": {"kind": "oracle", "cores": 1, "sample": res["desc"], "value": value,
+                                 "unit": "steps/s"},
+                "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+                "wall_s": time.time() - t_run}
+        print(json.dumps(line), flush=True)
+        return
+
+    if world > 1:
+        import torch
+        torch.distributed.init_process_group("nccl")
+    r = run_gpu(args, wl, rank, world)
+    if rank != 0:
+        if world > 1:
+            import torch
+            torch.distributed.destroy_process_group()
+        return
+    value = world * 1e3 / r["step_ms"]
+    e2e_value = world * 1e3 / r["e2e_ms"]
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        res = cpu_sample_subprocess(args.workload, wl["H"], 1, 41, 5)
+        sec = statistics.median(res["sec_per_step"])
+        cpu = {"value": 1.0 / sec, "unit": "steps/s", "cores": 1, "kind": "oracle", "sample": res["desc"]}
+    line = {
+        "metric": metric, "value": value, "unit": "steps/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": r["step_ms"], "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config,
+        "hbm_gbs_step": r["step_bytes"] / (r["step_ms"] * 1e-3) / 1e9,
+        "roofline": {"bound": "hbm", "kernel": "tree_attn_kernel<128>" if wl["D"] == 128 else "tree_attn_kernel<64>",
+                     "achieved": r["achieved"], "peak": r["peak"], "unit": "GB/s",
+                     "frac": r["achieved"] / r["peak"], "peak_source": f"{r['peak_kind']} (hbm_gbs)",
+                     "traffic": r["traffic"], "algorithmic_bytes_per_launch": r["attn_bytes"],
+                     "avg_launch_us": r["attn_ms"] * 1e3, "kernel_sha": r["sha"]},
+        "e2e": {"value": e2e_value, "unit": "steps/s", "h2d_bytes_per_step": r["h2d"],
+                "d2h_bytes_per_step": r["d2h"]},
+        "gpu_launches": r["launches"],
+        "clocks": r["clocks"],
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -281,13 +281,15 @@ def tree_accept(target_logits, draft_logits, tokens, parents, node_offsets, mode
     draft_logits[draft_row[v]] (identity when draft_row is None).
 
     Returns dict(path [B][*] tree-local node lists, accept_len [B],
-    bonus [B], min_margin): min_margin is the smallest relative decision
-    margin met (inf for GREEDY, whose decisions are exact comparisons).
+    bonus [B], accept_margin, sample_margin, min_margin): the smallest
+    relative margin of the accept tests, of the inverse-CDF draws, and of
+    both (inf for GREEDY, whose decisions are exact comparisons).
     """
     tokens = [int(t) for t in tokens]
     B = len(node_offsets) - 1
     paths, acc, bonus = [], [], []
-    min_margin = math.inf
+    acc_margin = math.inf
+    smp_margin = math.inf
     for b in range(B):
         lo, hi = int(node_offsets[b]), int(node_offsets[b + 1])
         par = [int(p) for p in parents[lo:hi]]
@@ -321,7 +323,7 @@ def tree_accept(target_logits, draft_logits, tokens, parents, node_offsets, mode
                     lhs, rhs = u * q[x], p[x]
                 scale = max(abs(lhs), abs(rhs))
                 if scale > 0:
-                    min_margin = min(min_margin, abs(lhs - rhs) / scale)
+                    acc_margin = min(acc_margin, abs(lhs - rhs) / scale)
                 if lhs < rhs:
                     nxt = c
                     break
@@ -340,7 +342,7 @@ def tree_accept(target_logits, draft_logits, tokens, parents, node_offsets, mode
                     q = q / qs if qs > 0 else np.zeros_like(q)
             if nxt is None:
                 t, m = sample_inverse_cdf(p, float(u_sample[gv]))
-                min_margin = min(min_margin, m)
+                smp_margin = min(smp_margin, m)
                 bonus.append(t)
                 break
             path.append(nxt)
@@ -348,7 +350,8 @@ def tree_accept(target_logits, draft_logits, tokens, parents, node_offsets, mode
         paths.append(path)
         acc.append(len(path) - 1)
     return dict(path=paths, accept_len=np.asarray(acc, np.int32),
-                bonus=np.asarray(bonus, np.int32), min_margin=min_margin)
+                bonus=np.asarray(bonus, np.int32), accept_margin=acc_margin,
+                sample_margin=smp_margin, min_margin=min(acc_margin, smp_margin))
 
 
 # ----------------------------------------------------------------------------

@@ -1,0 +1,137 @@
+// Host-side depth / width controller of ADT-Tree (Sec. 4.1 adjacent
+// initialisation, Eq. 2 bisectional adaptation, the bounds at the end of
+// Sec. 4.2, hyper-parameters of Sec. 5.1).  One object per image; no GPU.
+#include <cstdint>
+#include <new>
+#include <vector>
+
+#include "adt.h"
+
+struct adt_ctrl {
+  adt_ctrl_params p;
+  int32_t h, w;
+  std::vector<int32_t> d_grid, k_grid;  // (d, k) of the tree that emitted each position; 0 = not yet
+  bool have_alpha = false;
+  double alpha_prev = 0.0;
+  bool have_cur = false;
+  int32_t cur_d = 0, cur_k = 0;
+};
+
+namespace {
+
+constexpr uint64_t kGamma = 0x9E3779B97F4A7C15ull;
+
+// SplitMix64 (Steele, Lea, Flood 2014): one output for a state.
+uint64_t splitmix64(uint64_t state) {
+  uint64_t z = state + kGamma;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+uint64_t counter_draw(uint64_t seed, uint64_t counter) { return splitmix64(seed + counter * kGamma); }
+
+int32_t clamp(int32_t x, int32_t lo, int32_t hi) { return x < lo ? lo : (x > hi ? hi : x); }
+
+}  // namespace
+
+extern "C" {
+
+adt_status adt_ctrl_create(const adt_ctrl_params* params, int32_t grid_h, int32_t grid_w,
+                           adt_ctrl** out) {
+  if (!params || !out || grid_h < 1 || grid_w < 1) return ADT_ERR_INVALID_ARG;
+  const adt_ctrl_params& p = *params;
+  if (p.d_lo < 1 || p.d_hi < p.d_lo || p.k_lo < 1 || p.k_hi < p.k_lo || p.k_cap < p.k_hi) return ADT_ERR_INVALID_ARG;
+  if (p.l_d < 0 || p.l_k < 0 || p.d0 < 1 || p.k0 < 1 || p.fix_d < 0 || p.fix_k < 0) return ADT_ERR_INVALID_ARG;
+  if (p.init_mode != ADT_INIT_HORIZONTAL && p.init_mode != ADT_INIT_VERTICAL && p.init_mode != ADT_INIT_RANDOM)
+    return ADT_ERR_INVALID_ARG;
+  if (static_cast<int64_t>(grid_h) * grid_w > (int64_t{1} << 28)) return ADT_ERR_INVALID_ARG;
+  adt_ctrl* c = new (std::nothrow) adt_ctrl;
+  if (!c) return ADT_ERR_INVALID_ARG;
+  c->p = p;
+  c->h = grid_h;
+  c->w = grid_w;
+  try {
+    c->d_grid.assign(static_cast<size_t>(grid_h) * grid_w, 0);
+    c->k_grid.assign(static_cast<size_t>(grid_h) * grid_w, 0);
+  } catch (...) {
+    delete c;
+    return ADT_ERR_INVALID_ARG;
+  }
+  *out = c;
+  return ADT_OK;
+}
+
+void adt_ctrl_destroy(adt_ctrl* ctrl) { delete ctrl; }
+
+adt_status adt_ctrl_next(adt_ctrl* c, int32_t pos, int32_t* depth, int32_t* width) {
+  if (!c || !depth || !width) return ADT_ERR_INVALID_ARG;
+  const int32_t n = c->h * c->w;
+  if (pos < 0 || pos >= n) return ADT_ERR_INVALID_ARG;
+  const adt_ctrl_params& P = c->p;
+  const int32_t i = pos / c->w;
+  int32_t d, k;
+  // Adjacent initialisation (Sec. 4.1).
+  if (P.init_mode == ADT_INIT_RANDOM) {
+    d = P.d_lo + static_cast<int32_t>(counter_draw(P.seed, 2ull * static_cast<uint64_t>(pos)) %
+                                      static_cast<uint64_t>(P.d_hi - P.d_lo + 1));
+    k = P.k_lo + static_cast<int32_t>(counter_draw(P.seed, 2ull * static_cast<uint64_t>(pos) + 1) %
+                                      static_cast<uint64_t>(P.k_hi - P.k_lo + 1));
+  } else if (P.init_mode == ADT_INIT_VERTICAL && i >= 1 && c->d_grid[pos - c->w] > 0) {
+    d = c->d_grid[pos - c->w];
+    k = c->k_grid[pos - c->w];
+  } else if (pos >= 1 && c->d_grid[pos - 1] > 0) {
+    d = c->d_grid[pos - 1];
+    k = c->k_grid[pos - 1];
+  } else {
+    d = P.d0;
+    k = P.k0;
+  }
+  if (P.fix_d > 0) d = P.fix_d;
+  if (P.fix_k > 0) k = P.fix_k;
+  // Bisectional dynamic adaptation (Eq. 2).
+  if (c->have_alpha) {
+    if (c->alpha_prev >= P.beta) {
+      d += P.l_d;
+      k -= P.l_k;
+    } else {
+      d -= P.l_d;
+      k += P.l_k;
+    }
+  }
+  // Bounds (end of Sec. 4.2): width is restricted only when the adapted depth exceeds 1.
+  const bool restrict_k = P.clamp_k_always != 0 || d > 1;
+  d = clamp(d, P.d_lo, P.d_hi);
+  k = restrict_k ? clamp(k, P.k_lo, P.k_hi) : clamp(k, 1, P.k_cap);
+  c->cur_d = d;
+  c->cur_k = k;
+  c->have_cur = true;
+  *depth = d;
+  *width = k;
+  return ADT_OK;
+}
+
+adt_status adt_ctrl_update(adt_ctrl* c, int32_t pos, int32_t accept_len, int32_t* next_pos) {
+  if (!c || !c->have_cur) return ADT_ERR_INVALID_ARG;
+  const int32_t n = c->h * c->w;
+  if (pos < 0 || pos >= n || accept_len < 0 || accept_len > c->cur_d) return ADT_ERR_INVALID_ARG;
+  // alpha = accepted draft nodes / tree depth (Sec. 3.2 defines alpha = tau / d).
+  c->alpha_prev = static_cast<double>(accept_len) / static_cast<double>(c->cur_d);
+  c->have_alpha = true;
+  const int32_t end = pos + accept_len + 1 < n ? pos + accept_len + 1 : n;
+  for (int32_t t = pos; t < end; ++t) {
+    c->d_grid[t] = c->cur_d;
+    c->k_grid[t] = c->cur_k;
+  }
+  if (next_pos) *next_pos = pos + accept_len + 1;
+  return ADT_OK;
+}
+
+adt_status adt_ctrl_get(const adt_ctrl* c, int32_t pos, int32_t* depth, int32_t* width) {
+  if (!c || !depth || !width || pos < 0 || pos >= c->h * c->w) return ADT_ERR_INVALID_ARG;
+  *depth = c->d_grid[pos];
+  *width = c->k_grid[pos];
+  return ADT_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,584 @@
+// adt_tree_accept: the verification walk (Sec. 3.1, Eq. 1; greedy T = 0 and
+// sampling T = 1 as in Sec. 5.1).
+//
+// One thread-block cluster per tree.  The vocabulary is split into equal
+// slices, one per CTA of the cluster; a CTA keeps its slice of the current
+// node's target (and draft) row in shared memory.  Vocabulary-wide
+// quantities (argmax, max, sum of exponentials, residual mass, the CDF
+// offset of each slice) are block reductions whose per-CTA results are
+// published in shared memory and read by every CTA of the cluster through
+// distributed shared memory after a cluster barrier.  Every CTA sums the
+// published values in the same order, so all CTAs take identical decisions
+// without further communication.  p(x), q(x) of a child's token are read
+// from the owning CTA's slice.  The walk itself (children in ascending
+// index, one accept test each) is sequential, as the method defines it.
+#include <cooperative_groups.h>
+
+#include "adt_common.cuh"
+
+namespace cg = cooperative_groups;
+
+namespace {
+
+constexpr int kThreads = 512;
+constexpr int kMaxNodes = 1024;
+constexpr int kMaxCluster = 16;
+
+struct AcceptParams {
+  const float* target;
+  int64_t ldt;
+  const float* draft;
+  int64_t ldd;
+  const int32_t* drow;
+  const int32_t* tokens;
+  const int32_t* parents;
+  const int32_t* offs;
+  int B, V, max_nodes;
+  const float* ua;
+  const float* us;
+  int mode;
+  float T;
+  int use_T;
+  int32_t* path;
+  int max_path;
+  int32_t* alen;
+  int32_t* bonus;
+  unsigned* err;
+  int Vs;  // vocabulary slice per CTA (multiple of 4)
+};
+
+// Values a CTA publishes to its cluster; two copies alternate so that one
+// barrier per exchange suffices.
+struct Slot {
+  double d[2];
+  float f[2];
+  int i[2];
+};
+
+struct Shared {
+  Slot slot[2];
+  int par[kMaxNodes];
+  int tok[kMaxNodes];
+  int kids[kMaxNodes];
+  int path[kMaxNodes];
+  int rejected[kMaxNodes];
+  double dred[32];
+  float fred[32];
+  int ired[32];
+  int nkids;
+  int bad;
+  int found;
+  int last_pos;
+};
+
+struct Walker {
+  cg::cluster_group cl;
+  Shared* sh;
+  int rank, csize, parity;
+  __device__ Slot* publish_slot() { return &sh->slot[parity]; }
+  // Barrier, then return the published slot of CTA c (same parity).
+  __device__ const Slot* peer(int c) { return cl.map_shared_rank(&sh->slot[parity], c); }
+  __device__ void exchange() {
+    cl.sync();
+  }
+  __device__ void flip() { parity ^= 1; }
+};
+
+__device__ __forceinline__ bool better(float v, int i, float bv, int bi) {
+  return v > bv || (v == bv && i < bi);
+}
+
+// Block argmax over (value desc, index asc); all threads get the result.
+__device__ void block_argmax(float& v, int& idx, Shared* sh) {
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ov = __shfl_xor_sync(adt::kFullMask, v, o);
+    const int oi = __shfl_xor_sync(adt::kFullMask, idx, o);
+    if (better(ov, oi, v, idx)) {
+      v = ov;
+      idx = oi;
+    }
+  }
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  __syncthreads();
+  if (lane == 0) {
+    sh->fred[warp] = v;
+    sh->ired[warp] = idx;
+  }
+  __syncthreads();
+  v = lane < kThreads / 32 ? sh->fred[lane] : -INFINITY;
+  idx = lane < kThreads / 32 ? sh->ired[lane] : 0x7fffffff;
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ov = __shfl_xor_sync(adt::kFullMask, v, o);
+    const int oi = __shfl_xor_sync(adt::kFullMask, idx, o);
+    if (better(ov, oi, v, idx)) {
+      v = ov;
+      idx = oi;
+    }
+  }
+}
+
+// Loads this CTA's slice of a logit row (divided by T) into buf; entries
+// past V are -inf.
+__device__ void load_slice(const float* row, int lo, int cnt, int Vs, float* buf, const AcceptParams& p) {
+  for (int i = threadIdx.x * 4; i < Vs; i += kThreads * 4) {
+    float x[4];
+    if (i + 3 < cnt) {
+      const float4 v = __ldg(reinterpret_cast<const float4*>(row + lo + i));
+      x[0] = v.x; x[1] = v.y; x[2] = v.z; x[3] = v.w;
+    } else {
+      for (int e = 0; e < 4; ++e) x[e] = (i + e < cnt) ? __ldg(row + lo + i + e) : -INFINITY;
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      float y = x[e];
+      if (p.use_T && i + e < cnt) y = __fdiv_rn(y, p.T);
+      buf[i + e] = y;
+    }
+  }
+}
+
+// exp(x - M) in place over the slice; returns the block's sum (fp64 from
+// per-thread fp32 partials).
+__device__ double exp_in_place(float* buf, int Vs, float M, Shared* sh) {
+  float acc = 0.f;
+  for (int i = threadIdx.x; i < Vs; i += kThreads) {
+    const float e = expf(buf[i] - M);
+    buf[i] = e;
+    acc += e;
+  }
+  return adt::block_sum<kThreads, double>(static_cast<double>(acc), sh->dred);
+}
+
+__device__ float slice_max(const float* buf, int Vs, Shared* sh) {
+  float m = -INFINITY;
+  for (int i = threadIdx.x; i < Vs; i += kThreads) m = fmaxf(m, buf[i]);
+  return adt::block_max<kThreads>(m, sh->fred);
+}
+
+// Inverse-CDF draw over the (unnormalised, non-negative) distribution held
+// in the cluster's slices: smallest t with sum_{j<=t} w_j > u * sum_j w_j.
+// Returns the token id on every CTA.
+__device__ int cluster_sample(Walker& w, const float* buf, int lo, int cnt, double u, Shared* sh) {
+  // 1. per-CTA slice totals (each thread owns a contiguous run), published.
+  const int per = (cnt + kThreads - 1) / kThreads;
+  const int b0 = min(cnt, static_cast<int>(threadIdx.x) * per), b1 = min(cnt, b0 + per);
+  double run = 0.0;
+  int last_pos = -1;
+  for (int i = b0; i < b1; ++i) {
+    run += buf[i];
+    if (buf[i] > 0.f) last_pos = i;
+  }
+  const double tot = adt::block_sum<kThreads, double>(run, sh->dred);
+  if (threadIdx.x == 0) w.publish_slot()->d[0] = tot;
+  w.exchange();
+  double grand = 0.0, base = 0.0;
+  for (int c = 0; c < w.csize; ++c) {
+    const double t = w.peer(c)->d[0];
+    if (c < w.rank) base += t;
+    grand += t;
+  }
+  const double target = u * grand;
+  // Owner: first CTA whose cumulative total passes the target; else the last
+  // CTA with mass.
+  int owner = -1, last_nz = -1;
+  {
+    double acc = 0.0;
+    for (int c = 0; c < w.csize; ++c) {
+      const double t = w.peer(c)->d[0];
+      if (owner < 0 && acc + t > target) owner = c;
+      if (t > 0.0) last_nz = c;
+      acc += t;
+    }
+    if (owner < 0) owner = last_nz < 0 ? 0 : last_nz;
+  }
+  w.flip();
+  int result_local = -1;
+  if (w.rank == owner) {
+    // exclusive scan of the per-thread runs
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    double incl = run;
+    for (int o = 1; o < 32; o <<= 1) {
+      const double y = __shfl_up_sync(adt::kFullMask, incl, o);
+      if (lane >= o) incl += y;
+    }
+    __syncthreads();
+    if (lane == 31) sh->dred[warp] = incl;
+    if (threadIdx.x == 0) {
+      sh->found = 0x7fffffff;
+      sh->last_pos = -1;
+    }
+    __syncthreads();
+    double wbase = 0.0;
+    for (int j = 0; j < warp; ++j) wbase += sh->dred[j];
+    double acc = base + wbase + incl - run;
+    if (last_pos >= 0) atomicMax(&sh->last_pos, last_pos);
+    for (int i = b0; i < b1; ++i) {
+      const double wv = buf[i];
+      acc += wv;
+      if (acc > target && wv > 0.0) {
+        atomicMin(&sh->found, i);
+        break;
+      }
+    }
+    __syncthreads();
+    int t = sh->found;
+    if (t == 0x7fffffff) t = sh->last_pos < 0 ? 0 : sh->last_pos;
+    result_local = lo + t;
+    if (threadIdx.x == 0) w.publish_slot()->i[0] = result_local;
+  }
+  w.exchange();
+  const int res = w.peer(owner)->i[0];
+  w.flip();
+  return res;
+}
+
+__global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) {
+  extern __shared__ __align__(16) float dyn[];
+  __shared__ Shared sh;
+  cg::cluster_group cl = cg::this_cluster();
+  Walker w{cl, &sh, static_cast<int>(cl.block_rank()), static_cast<int>(cl.num_blocks()), 0};
+  const int b = blockIdx.x / w.csize;
+  const int tid = threadIdx.x;
+  float* pbuf = dyn;
+  float* qbuf = dyn + p.Vs;
+  const int lo = w.rank * p.Vs;
+  const int cnt = max(0, min(p.Vs, p.V - lo));
+
+  const int node0 = p.offs[b];
+  const int n = p.offs[b + 1] - node0;
+  if (tid == 0) sh.bad = (n < 1 || n > p.max_nodes) ? 1 : 0;
+  __syncthreads();
+  if (!sh.bad) {
+    for (int i = tid; i < n; i += kThreads) {
+      const int pr = p.parents[node0 + i];
+      sh.par[i] = pr;
+      sh.tok[i] = p.tokens[node0 + i];
+      if ((i == 0) != (pr < 0) || pr >= i) sh.bad = 1;
+    }
+  }
+  __syncthreads();
+  if (sh.bad) {
+    if (w.rank == 0 && tid == 0) {
+      adt::raise_error(p.err, ADT_DEVERR_BAD_TREE);
+      p.alen[b] = 0;
+      p.bonus[b] = 0;
+      for (int i = 0; i < p.max_path; ++i) p.path[static_cast<int64_t>(b) * p.max_path + i] = i == 0 ? 0 : -1;
+    }
+    cl.sync();
+    return;
+  }
+
+  int v = 0, plen = 1;
+  if (tid == 0) sh.path[0] = 0;
+  int bonus = 0;
+  for (int step = 0; step < n; ++step) {
+    // children of v, ascending
+    __syncthreads();
+    if (tid == 0) sh.nkids = 0;
+    __syncthreads();
+    for (int base = 0; base < n; base += kThreads) {
+      const int i = base + tid;
+      const bool f = i < n && sh.par[i] == v;
+      const unsigned bal = __ballot_sync(adt::kFullMask, f);
+      const int lane = tid & 31, warp = tid >> 5;
+      if (lane == 0) sh.ired[warp] = __popc(bal);
+      __syncthreads();
+      int before = 0;
+      for (int j = 0; j < warp; ++j) before += sh.ired[j];
+      if (f) sh.kids[sh.nkids + before + __popc(bal & ((1u << lane) - 1u))] = i;
+      __syncthreads();
+      if (tid == 0) {
+        int t = 0;
+        for (int j = 0; j < kThreads / 32; ++j) t += sh.ired[j];
+        sh.nkids += t;
+      }
+      __syncthreads();
+    }
+    const int nk = sh.nkids;
+    const int gv = node0 + v;
+    const float* trow = p.target + static_cast<int64_t>(gv) * p.ldt;
+
+    if (p.mode == ADT_ACCEPT_GREEDY) {
+      float bv = -INFINITY;
+      int bi = 0x7fffffff;
+      for (int i = tid; i < cnt; i += kThreads) {
+        const float x = __ldg(trow + lo + i);
+        if (better(x, lo + i, bv, bi)) {
+          bv = x;
+          bi = lo + i;
+        }
+      }
+      block_argmax(bv, bi, &sh);
+      if (tid == 0) {
+        w.publish_slot()->f[0] = bv;
+        w.publish_slot()->i[0] = bi;
+      }
+      w.exchange();
+      float gvv = -INFINITY;
+      int g = 0x7fffffff;
+      for (int c = 0; c < w.csize; ++c) {
+        const Slot* s = w.peer(c);
+        if (better(s->f[0], s->i[0], gvv, g)) {
+          gvv = s->f[0];
+          g = s->i[0];
+        }
+      }
+      w.flip();
+      int nxt = -1;
+      for (int j = 0; j < nk; ++j) {
+        if (sh.tok[sh.kids[j]] == g) {
+          nxt = sh.kids[j];
+          break;
+        }
+      }
+      if (nxt < 0) {
+        bonus = g;
+        break;
+      }
+      if (tid == 0) sh.path[plen] = nxt;
+      ++plen;
+      v = nxt;
+      continue;
+    }
+
+    // ---- sampling modes: p = softmax(target row / T) in the slices.
+    const bool spec = p.mode == ADT_ACCEPT_SPEC;
+    const bool need_q = spec && nk > 0;
+    load_slice(trow, lo, cnt, p.Vs, pbuf, p);
+    if (need_q) {
+      const int64_t dr = p.drow ? p.drow[gv] : gv;
+      load_slice(p.draft + dr * p.ldd, lo, cnt, p.Vs, qbuf, p);
+    }
+    __syncthreads();
+    const float mp = slice_max(pbuf, p.Vs, &sh);
+    const float mq = need_q ? slice_max(qbuf, p.Vs, &sh) : 0.f;
+    if (tid == 0) {
+      w.publish_slot()->f[0] = mp;
+      w.publish_slot()->f[1] = mq;
+    }
+    w.exchange();
+    float Mp = -INFINITY, Mq = -INFINITY;
+    for (int c = 0; c < w.csize; ++c) {
+      Mp = fmaxf(Mp, w.peer(c)->f[0]);
+      Mq = fmaxf(Mq, w.peer(c)->f[1]);
+    }
+    w.flip();
+    const double sp_loc = exp_in_place(pbuf, p.Vs, Mp, &sh);
+    const double sq_loc = need_q ? exp_in_place(qbuf, p.Vs, Mq, &sh) : 0.0;
+    if (tid == 0) {
+      w.publish_slot()->d[0] = sp_loc;
+      w.publish_slot()->d[1] = sq_loc;
+    }
+    w.exchange();
+    double Sp = 0.0, Sq = 0.0;
+    for (int c = 0; c < w.csize; ++c) {
+      Sp += w.peer(c)->d[0];
+      Sq += w.peer(c)->d[1];
+    }
+    w.flip();
+    if (spec && need_q) {
+      // normalise both slices (fp32)
+      const float ip = static_cast<float>(1.0 / Sp), iq = static_cast<float>(1.0 / Sq);
+      for (int i = tid; i < p.Vs; i += kThreads) {
+        pbuf[i] *= ip;
+        qbuf[i] *= iq;
+      }
+      w.exchange();  // slices final before any peer reads them
+      w.flip();
+    }
+
+    int nxt = -1;
+    double e_rej = 0.0;  // SPEC_DET: rejected unnormalised mass
+    int nrej = 0;
+    for (int j = 0; j < nk; ++j) {
+      const int c = sh.kids[j];
+      const int x = sh.tok[c];
+      if (x < 0 || x >= p.V) {
+        if (w.rank == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_BAD_INDEX);
+        continue;
+      }
+      const int owner = x / p.Vs, off = x - owner * p.Vs;
+      const double u = static_cast<double>(p.ua[node0 + c]);
+      bool acc;
+      if (!spec) {
+        bool dup = false;
+        for (int r = 0; r < nrej; ++r) dup |= sh.rejected[r] == x;
+        const double ex = dup ? 0.0 : static_cast<double>(*cl.map_shared_rank(pbuf + off, owner));
+        const double denom = Sp - e_rej;
+        const double px = denom > 0.0 ? ex / denom : 0.0;
+        acc = u < px;
+        if (!acc && !dup) {
+          e_rej += ex;
+          if (tid == 0) sh.rejected[nrej] = x;
+          ++nrej;
+          __syncthreads();
+        }
+      } else {
+        const double px = *cl.map_shared_rank(pbuf + off, owner);
+        const double qx = *cl.map_shared_rank(qbuf + off, owner);
+        acc = u * qx < px;
+        if (!acc) {
+          // residual: p <- max(0, p - q)/Z (kept if Z = 0); q(x) <- 0, q <- q/sum
+          float zl = 0.f, ql = 0.f;
+          for (int i = tid; i < p.Vs; i += kThreads) {
+            zl += fmaxf(pbuf[i] - qbuf[i], 0.f);
+            ql += (lo + i == x) ? 0.f : qbuf[i];
+          }
+          const double zb = adt::block_sum<kThreads, double>(static_cast<double>(zl), sh.dred);
+          const double qb = adt::block_sum<kThreads, double>(static_cast<double>(ql), sh.dred);
+          if (tid == 0) {
+            w.publish_slot()->d[0] = zb;
+            w.publish_slot()->d[1] = qb;
+          }
+          w.exchange();  // also: every peer has finished reading px, qx
+          double Z = 0.0, Qs = 0.0;
+          for (int cc = 0; cc < w.csize; ++cc) {
+            Z += w.peer(cc)->d[0];
+            Qs += w.peer(cc)->d[1];
+          }
+          w.flip();
+          const float iz = Z > 0.0 ? static_cast<float>(1.0 / Z) : 0.f;
+          const float iqs = Qs > 0.0 ? static_cast<float>(1.0 / Qs) : 0.f;
+          for (int i = tid; i < p.Vs; i += kThreads) {
+            const float pi = pbuf[i], qi = qbuf[i];
+            if (Z > 0.0) pbuf[i] = fmaxf(pi - qi, 0.f) * iz;
+            qbuf[i] = (lo + i == x) ? 0.f : qi * iqs;
+          }
+          w.exchange();  // updated slices visible before the next read
+          w.flip();
+        }
+      }
+      if (acc) {
+        nxt = c;
+        break;
+      }
+    }
+    if (nxt >= 0) {
+      if (tid == 0) sh.path[plen] = nxt;
+      ++plen;
+      v = nxt;
+      continue;
+    }
+    // bonus from the current (residual) p
+    if (!spec && nrej > 0) {
+      __syncthreads();
+      for (int r = 0; r < nrej; ++r) {
+        const int x = sh.rejected[r];
+        if (x >= lo && x < lo + cnt && tid == 0) pbuf[x - lo] = 0.f;
+      }
+    }
+    __syncthreads();
+    bonus = cluster_sample(w, pbuf, lo, cnt, static_cast<double>(p.us[gv]), &sh);
+    break;
+  }
+
+  __syncthreads();
+  if (w.rank == 0 && tid == 0) {
+    int64_t o = static_cast<int64_t>(b) * p.max_path;
+    if (plen > p.max_path) adt::raise_error(p.err, ADT_DEVERR_BAD_PATH);
+    for (int i = 0; i < p.max_path; ++i) p.path[o + i] = i < plen ? sh.path[i] : -1;
+    p.alen[b] = min(plen, p.max_path) - 1;
+    p.bonus[b] = bonus;
+  }
+  cl.sync();  // no CTA leaves while a peer may still read its shared memory
+}
+
+int cluster_size_for(int V) { return V <= 131072 ? 8 : 16; }
+
+int slice_for(int V, int cs) {
+  int vs = (V + cs - 1) / cs;
+  return (vs + 3) / 4 * 4;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t adt_tree_accept_workspace_size(int32_t B, int32_t V) {
+  (void)B;
+  (void)V;
+  return 0;
+}
+
+adt_status adt_tree_accept(const float* target_logits, int64_t ld_target,
+                           const float* draft_logits, int64_t ld_draft, const int32_t* draft_row,
+                           const int32_t* tokens, const int32_t* parents,
+                           const int32_t* node_offsets, int32_t B, int32_t V, int32_t max_nodes,
+                           const float* u_accept, const float* u_sample, adt_accept_mode mode,
+                           float temperature, int32_t* path, int32_t max_path,
+                           int32_t* accept_len, int32_t* bonus_token, void* workspace,
+                           size_t workspace_bytes, void* stream) {
+  (void)workspace;
+  (void)workspace_bytes;
+  ADT_REQUIRE(target_logits && tokens && parents && node_offsets && path && accept_len && bonus_token);
+  ADT_REQUIRE(mode == ADT_ACCEPT_GREEDY || mode == ADT_ACCEPT_SPEC || mode == ADT_ACCEPT_SPEC_DET);
+  ADT_REQUIRE(B >= 1 && V >= 1 && V <= 262144 && max_nodes >= 1 && max_path >= 1);
+  if (max_nodes > kMaxNodes) return ADT_ERR_UNSUPPORTED;
+  ADT_REQUIRE(ld_target >= V && ld_target % 4 == 0 && adt::aligned16(target_logits));
+  if (mode != ADT_ACCEPT_GREEDY) {
+    ADT_REQUIRE(u_accept && u_sample);
+    ADT_REQUIRE(temperature > 0.f && temperature < 1e30f);
+  }
+  if (mode == ADT_ACCEPT_SPEC) {
+    ADT_REQUIRE(draft_logits && ld_draft >= V && ld_draft % 4 == 0 && adt::aligned16(draft_logits));
+  }
+  adt::DeviceInfo info;
+  adt_status st = adt::device_info(&info);
+  if (st != ADT_OK) return st;
+  const int cs = cluster_size_for(V);
+  const int vs = slice_for(V, cs);
+  const size_t smem = static_cast<size_t>(vs) * sizeof(float) * (mode == ADT_ACCEPT_SPEC ? 2 : 1);
+  if (smem + sizeof(Shared) > static_cast<size_t>(info.max_smem_optin)) return ADT_ERR_UNSUPPORTED;
+  static int configured_smem[64];  // largest dynamic smem already allowed, per device
+  static int configured_np[64];
+  const int dev = info.device & 63;
+  if (configured_smem[dev] < static_cast<int>(smem)) {
+    ADT_CUDA_TRY(cudaFuncSetAttribute(accept_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      static_cast<int>(smem)));
+    configured_smem[dev] = static_cast<int>(smem);
+  }
+  if (cs > 8 && !configured_np[dev]) {
+    ADT_CUDA_TRY(cudaFuncSetAttribute(accept_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1));
+    configured_np[dev] = 1;
+  }
+  AcceptParams p;
+  p.target = target_logits;
+  p.ldt = ld_target;
+  p.draft = draft_logits;
+  p.ldd = ld_draft;
+  p.drow = draft_row;
+  p.tokens = tokens;
+  p.parents = parents;
+  p.offs = node_offsets;
+  p.B = B;
+  p.V = V;
+  p.max_nodes = max_nodes;
+  p.ua = u_accept;
+  p.us = u_sample;
+  p.mode = static_cast<int>(mode);
+  p.T = temperature;
+  p.use_T = mode != ADT_ACCEPT_GREEDY && temperature != 1.0f;
+  p.path = path;
+  p.max_path = max_path;
+  p.alen = accept_len;
+  p.bonus = bonus_token;
+  p.err = info.error_word;
+  p.Vs = vs;
+
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(cs * B), 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = adt::as_stream(stream);
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cs;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, accept_kernel, p));
+  return adt::launch_status();
+}
+
+}  // extern "C"

@@ -153,3 +153,25 @@ def acceptance_map(h: int, w: int, seed: int, n_blobs: int = 6, lo: float = 0.15
         acc += amp * np.exp(-((yy - cy) ** 2 + (xx - cx) ** 2) / (2 * s * s))
     acc = (acc - acc.min()) / max(acc.max() - acc.min(), 1e-12)
     return lo + (hi - lo) * acc
+
+
+def step_inputs(layers, H, Hkv, D, V, kv_len, depth, width, n_nodes, lmax, seed, logit_std=3.0):
+    """Host inputs of one verify step (all seeded): caches and tree
+    projections bf16 ~ N(0, 1); draft rows per image and layer fp32
+    ~ N(0, logit_std^2); target rows ~ N(0, logit_std^2); uniforms; root
+    tokens.  n_nodes[b] is the tree size of image b."""
+    Bn = len(kv_len)
+    ntot = int(sum(n_nodes))
+    out = dict(
+        k_cache=bf16_normal((layers, Bn, Hkv, lmax, D), seed, "k_cache"),
+        v_cache=bf16_normal((layers, Bn, Hkv, lmax, D), seed, "v_cache"),
+        q=bf16_normal((layers, ntot, H, D), seed, "q"),
+        k_tree=bf16_normal((layers, ntot, Hkv, D), seed, "k_tree"),
+        v_tree=bf16_normal((layers, ntot, Hkv, D), seed, "v_tree"),
+        draft_rows=[f32_normal((depth[b], width[b], V), seed, f"draft{b}", std=logit_std) for b in range(Bn)],
+        target=f32_normal((ntot, V), seed, "target", std=logit_std),
+        u_accept=uniforms(ntot, seed, "u_accept"),
+        u_sample=uniforms(ntot, seed, "u_sample"),
+        root_token=rng(seed, "root").integers(0, V, size=Bn).astype(np.int32),
+    )
+    return out

@@ -1,0 +1,81 @@
+"""GPU tree attention vs the oracle, element by element (tolerance: max-abs
+1e-2 and normwise 2e-2 on bf16 inputs), over the workload shapes of the
+7B-class and LlamaGen-class models and the edge cases."""
+import numpy as np
+import pytest
+
+from gpu_cases import AttnCase, assert_attention_close, ensure_built
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    ensure_built()
+
+
+CASES = [
+    # sizes, kv_lens, H, Hkv, D
+    ([26], [512], 8, 8, 64),              # single verify step, batch 1, 26-node tree
+    ([64], [696], 20, 20, 64),            # LlamaGen-XL-shaped layer, 64 nodes, 120 + 576 prefix
+    ([16], [120], 20, 20, 64),            # LlamaGen-XL, text prefix only
+    ([33, 7, 1, 64], [63, 64, 65, 0], 4, 4, 128),  # ragged batch, tile edges, empty prefix
+    ([12, 5], [700, 1], 8, 2, 128),       # grouped kv heads
+    ([1], [300], 4, 4, 64),               # single node = ordinary decode attention
+]
+
+
+@pytest.mark.parametrize("sizes,kv,H,Hkv,D", CASES)
+def test_attention_matches_oracle(sizes, kv, H, Hkv, D):
+    case = AttnCase(sizes, kv, H, Hkv, D, seed=101 + sum(sizes))
+    got, lse, _ = case.run_gpu()
+    ref, ref_lse = case.run_oracle()
+    assert_attention_close(got, ref)
+    assert np.abs(lse - ref_lse).max() < 2e-3
+
+
+def test_chain_tree_matches_oracle():
+    case = AttnCase([64], [257], 4, 4, 128, seed=7, chain=True)
+    got, _, _ = case.run_gpu()
+    ref, _ = case.run_oracle()
+    assert_attention_close(got, ref)
+
+
+def test_7b_shape_one_layer_full_size():
+    """KV 2400, 32 heads x 128, 64-node tree: the launch configuration the
+    benchmark times (one layer; every layer is the same call)."""
+    case = AttnCase([64], [2400], 32, 32, 128, seed=2024, lmax=2400 + 64)
+    got, lse, _ = case.run_gpu(max_kv=2400 + 64)
+    ref, ref_lse = case.run_oracle()
+    assert_attention_close(got, ref)
+    assert np.abs(lse - ref_lse).max() < 2e-3
+
+
+def test_batch_of_eight_ragged_prefixes():
+    g = np.random.default_rng(5)
+    kv = g.integers(600, 2401, size=8).tolist()
+    sizes = g.integers(8, 65, size=8).tolist()
+    case = AttnCase(sizes, kv, 8, 8, 128, seed=77, max_depth=10, max_children=8)
+    got, _, _ = case.run_gpu(max_nodes=64, max_kv=2400)
+    ref, _ = case.run_oracle()
+    assert_attention_close(got, ref)
+
+
+def test_workspace_reuse_and_repeat_is_deterministic():
+    case = AttnCase([26], [512], 8, 8, 64, seed=3)
+    a, la, ws = case.run_gpu()
+    b, lb, _ = case.run_gpu()
+    assert np.array_equal(a, b) and np.array_equal(la, lb)
+    # the ticket counters are back at zero after every call
+    assert int(ws[-256:].cpu().sum()) == 0
+
+
+def test_bad_tree_sets_device_error():
+    from paper_2512_21857_gb300 import binding as B
+    case = AttnCase([5], [10], 2, 2, 64, seed=1)
+    case.tb.parents[3] = 4  # parent after child
+    B.adt_get_device_error()
+    case.run_gpu()
+    bits = B.adt_get_device_error()
+    assert bits & B.DEVERR_BAD_TREE
+    assert B.adt_get_device_error() == 0

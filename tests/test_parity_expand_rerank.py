@@ -1,0 +1,186 @@
+"""GPU draft-tree expansion and rerank vs the oracle.  Token ids, parents,
+candidate indices and depths must match bit for bit; log-probabilities and
+scores (fp32 outputs of an fp64 formula with fp32 exponentials inside the
+normaliser) within 5e-5.  Where the oracle's own selection has a near tie
+(score gap < 1e-5), the GPU selection is checked for validity instead."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_cases import ensure_built, f32, grow_candidates_gpu, i32
+from paper_2512_21857_gb300 import binding as B
+from paper_2512_21857_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+TOL = 5e-5
+TIE = 1e-5
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    ensure_built()
+
+
+def run_expand(logits, fscore, fid, k, keep, T=1.0, base=0):
+    F, V = logits.shape
+    dev = "cuda"
+    ws = B.zeroed_workspace(B.adt_tree_expand_workspace_size(F, V, k))
+    out = dict(child_token=torch.empty(F * k, dtype=torch.int32, device=dev),
+               child_logp=torch.empty(F * k, dtype=torch.float32, device=dev),
+               child_score=torch.empty(F * k, dtype=torch.float32, device=dev),
+               child_parent=torch.empty(F * k, dtype=torch.int32, device=dev))
+    keep_idx = torch.empty(keep, dtype=torch.int32, device=dev)
+    ns = torch.empty(keep, dtype=torch.float32, device=dev)
+    nid = torch.empty(keep, dtype=torch.int32, device=dev)
+    B.adt_tree_expand(f32(logits), f32(fscore), None if fid is None else i32(fid), F=F, V=V, k_child=k,
+                      k_keep=keep, temperature=T, child_id_base=base, keep_idx=keep_idx, next_score=ns,
+                      next_id=nid, workspace=ws, **out)
+    torch.cuda.synchronize()
+    res = {kk: v.cpu().numpy() for kk, v in out.items()}
+    res.update(keep_idx=keep_idx.cpu().numpy(), next_score=ns.cpu().numpy(), next_id=nid.cpu().numpy())
+    # the completion counters (end of the workspace) are back at zero
+    assert int(ws[-256:].cpu().sum()) == 0
+    return res, ws
+
+
+def near_tie(scores, count):
+    s = np.sort(np.asarray(scores, np.float64))[::-1][:count + 1]
+    return len(s) > 1 and np.min(np.abs(np.diff(s))) < TIE
+
+
+def check_expand(got, ref, k_keep):
+    assert np.array_equal(got["child_token"], ref["child_token"])
+    assert np.array_equal(got["child_parent"], ref["child_parent"])
+    assert np.abs(got["child_logp"] - ref["child_logp"]).max() <= TOL
+    assert np.abs(got["child_score"] - ref["child_score"]).max() <= TOL
+    if near_tie(ref["child_score"], k_keep):
+        # valid selection w.r.t. the GPU's own scores
+        order = sorted(range(len(got["child_score"])), key=lambda c: (-float(got["child_score"][c]), c))
+        assert got["keep_idx"].tolist() == order[:k_keep]
+    else:
+        assert np.array_equal(got["keep_idx"], ref["keep_idx"])
+        assert np.array_equal(got["next_id"], ref["next_id"])
+    assert np.array_equal(got["next_score"], got["child_score"][got["keep_idx"]])
+
+
+@pytest.mark.parametrize("F,V,k,keep,T", [
+    (1, 65536, 8, 8, 1.0),       # first layer of the 7B-shape tree
+    (8, 65536, 8, 8, 1.0),       # later layers
+    (13, 16384, 13, 13, 1.0),    # Anole width bound
+    (39, 16384, 39, 39, 1.0),    # LlamaGen width bound
+    (4, 100, 64, 100, 1.0),      # k > chunk rows, k_keep > 64
+    (3, 4099, 5, 7, 0.7),        # ragged last chunk, temperature
+    (2, 7, 7, 14, 1.0),          # V == k
+])
+def test_expand_matches_oracle(F, V, k, keep, T):
+    seed = F * 1000 + V
+    logits = synth.f32_normal((F, V), seed, "logits", std=3.0)
+    fscore = synth.f32_normal((F,), seed, "fs", std=1.0) - 2.0
+    fid = np.arange(F, dtype=np.int32) * 3 + 1
+    got, _ = run_expand(logits, fscore, fid, k, keep, T, base=17)
+    ref = oracle.tree_expand(logits, fscore, k, keep, temperature=T, frontier_id=fid, child_id_base=17)
+    check_expand(got, ref, keep)
+
+
+def test_expand_ties_take_lowest_index():
+    V = 20000
+    logits = np.zeros((2, V), np.float32)
+    logits[0, 5000:5003] = 1.0      # three-way tie at the top
+    logits[0, 17] = -0.0            # -0.0 equals +0.0
+    logits[1, :] = np.float32(2.5)  # a row of ties: lowest indices win
+    fscore = np.array([0.0, -1.0], np.float32)
+    got, _ = run_expand(logits, fscore, None, 6, 5)
+    ref = oracle.tree_expand(logits, fscore, 6, 5)
+    assert got["child_token"][:6].tolist() == [5000, 5001, 5002, 0, 1, 2]
+    assert got["child_token"][6:].tolist() == [0, 1, 2, 3, 4, 5]
+    check_expand(got, ref, 5)
+
+
+def test_expand_repeated_calls_reuse_workspace():
+    logits = synth.f32_normal((8, 65536), 9, "l")
+    fs = np.zeros(8, np.float32)
+    a, _ = run_expand(logits, fs, None, 8, 8)
+    b, _ = run_expand(logits, fs, None, 8, 8)
+    for key in a:
+        assert np.array_equal(a[key], b[key])
+
+
+def _oracle_grow(draft_rows, k, depth, root_token, n_nodes):
+    tok, sc, par = [], [], []
+    fscore = np.zeros(1, np.float32)
+    fid = np.array([-1], np.int32)
+    ties = False
+    for d in range(depth):
+        F = len(fscore)
+        res = oracle.tree_expand(draft_rows[d][:F], fscore, k, min(k, F * k), frontier_id=fid,
+                                 child_id_base=len(tok))
+        ties |= near_tie(res["child_score"], min(k, F * k))
+        tok += res["child_token"].tolist()
+        sc += res["child_score"].tolist()
+        par += res["child_parent"].tolist()
+        fscore, fid = res["next_score"], res["next_id"]
+    n = min(n_nodes, len(tok) + 1)
+    ties |= near_tie(sc, n - 1)
+    tree = oracle.tree_rerank(tok, np.array(sc, np.float32), par, root_token, n)
+    return tree, np.array(tok), np.array(sc, np.float32), np.array(par), ties
+
+
+@pytest.mark.parametrize("V,k,depth,n", [(65536, 8, 6, 64), (16384, 10, 5, 64), (16384, 4, 9, 30),
+                                         (1000, 3, 2, 12)])
+def test_grown_tree_matches_oracle(V, k, depth, n):
+    """d-hat expand calls chained on the device, then the final rerank: the
+    draft phase of one ADT-Tree step (Sec. 3.1, Fig. 5, Eq. 4)."""
+    seed = V + k * 10 + depth
+    rows = [synth.f32_normal((k, V), seed, f"draft{d}", std=3.0) for d in range(depth)]
+    g = grow_candidates_gpu(rows, k, depth, 4242, n)
+    tree, tok, sc, par, ties = _oracle_grow(rows, k, depth, 4242, n)
+    assert not ties, "near tie in the seeded draft rows: pick another seed"
+    assert np.array_equal(g["pool_token"], tok)
+    assert np.array_equal(g["pool_parent"], par)
+    assert np.abs(g["pool_score"] - sc).max() <= TOL
+    for key in ("tokens", "parents", "cand_index", "depth"):
+        assert np.array_equal(g["tree"][key], tree[key]), key
+
+
+def _random_pool(C, seed):
+    """A valid depth-major candidate pool: parents precede children and a
+    child's score never exceeds its parent's."""
+    g = np.random.default_rng(seed)
+    tok = g.integers(0, 50000, C).astype(np.int32)
+    par = np.full(C, -1, np.int32)
+    sc = np.zeros(C, np.float32)
+    layer_start, layer = 0, 0
+    i = 0
+    while i < C:
+        width = int(g.integers(1, 40))
+        prev = list(range(layer_start, i)) if layer else []
+        start = i
+        for _ in range(width):
+            if i >= C:
+                break
+            if prev:
+                p = int(g.choice(prev))
+                par[i] = p
+                sc[i] = np.float32(sc[p] - np.float32(abs(g.standard_normal()) + 1e-3))
+            else:
+                sc[i] = np.float32(-abs(g.standard_normal()))
+            i += 1
+        layer_start, layer = start, layer + 1
+    return tok, sc, par
+
+
+@pytest.mark.parametrize("C,n", [(328, 64), (1534, 64), (5000, 4096), (9, 10), (70, 1)])
+def test_rerank_matches_oracle(C, n):
+    tok, sc, par = _random_pool(C, seed=C + n)
+    dev = "cuda"
+    res = dict(tokens=torch.empty(n, dtype=torch.int32, device=dev),
+               parents=torch.empty(n, dtype=torch.int32, device=dev),
+               cand_index=torch.empty(n, dtype=torch.int32, device=dev),
+               depth=torch.empty(n, dtype=torch.int32, device=dev))
+    ws = B.zeroed_workspace(B.adt_tree_rerank_workspace_size(C))
+    B.adt_tree_rerank(i32(tok), f32(sc), i32(par), C, i32([7]), n, workspace=ws, **res)
+    torch.cuda.synchronize()
+    ref = oracle.tree_rerank(tok, sc, par, 7, n)
+    for key in res:
+        assert np.array_equal(res[key].cpu().numpy(), ref[key]), key
