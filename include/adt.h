@@ -34,8 +34,12 @@
  *   - Workspace: a call that needs scratch memory takes (workspace,
  *     workspace_bytes); size it with the matching *_workspace_size() query.
  *     The workspace must be zero-filled once before its first use; every
- *     call leaves its counters at zero again when it completes.  Calls that
- *     share a workspace must not overlap in time.
+ *     call leaves its completion counters (kept at fixed offsets at the
+ *     start of the workspace) at zero again when it completes, so one
+ *     workspace can serve any sequence of calls of the same entry point,
+ *     of any shape, if it is as large as the largest query.  A workspace
+ *     serves one entry point only, and calls that share it must not overlap
+ *     in time.  After a call that reported a device error, zero it again.
  *   - bf16 tensors are raw IEEE bfloat16 bit patterns (adt_bf16).
  *   - Tree layout: B trees packed back to back.  node_offsets[b] ..
  *     node_offsets[b+1]-1 are the global indices of tree b's nodes; within a

@@ -181,6 +181,8 @@ def adt_tree_expand(logits, frontier_score, frontier_id, *, F, V, k_child, k_kee
     _expect(frontier_score, torch.float32, "frontier_score")
     if logits.dtype != torch.float32 or logits.stride(-1) != 1:
         raise TypeError("logits: fp32 rows with unit inner stride")
+    if logits.dim() != 2:
+        raise ValueError("logits: [F, V] rows")
     ld = logits.stride(0) if ld is None else ld
     st = lib().adt_tree_expand(_ptr(logits), ld, _ptr(frontier_score), _ptr(frontier_id), F, V, k_child, k_keep,
                                float(temperature), int(child_id_base), _ptr(child_token), _ptr(child_logp),

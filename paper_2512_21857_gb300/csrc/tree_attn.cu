@@ -395,17 +395,22 @@ int choose_splits(int sm_count, int B, int H, int D, int max_kv) {
   return s;
 }
 
+// Workspace layout.  The per-(tree, head) completion tickets sit at fixed
+// offsets at the start (room for kMaxBH pairs), so calls of any shape can
+// share one workspace; the partials after them are rewritten before use.
+constexpr int kMaxBH = 65536;
+
 struct WsLayout {
-  size_t part_o, part_ml, tickets, total;
+  size_t tickets, part_ml, part_o, total;
 };
 
 WsLayout ws_layout(int B, int H, int D, int splits) {
   WsLayout w{};
   const size_t bhs = static_cast<size_t>(B) * H * splits;
-  w.part_o = 0;
-  w.part_ml = adt::align_up(w.part_o + bhs * kMaxNodes * D * sizeof(float), 256);
-  w.tickets = adt::align_up(w.part_ml + bhs * kMaxNodes * sizeof(float2), 256);
-  w.total = adt::align_up(w.tickets + static_cast<size_t>(B) * H * sizeof(unsigned), 256);
+  w.tickets = 0;
+  w.part_ml = adt::align_up(static_cast<size_t>(kMaxBH) * sizeof(unsigned), 256);
+  w.part_o = adt::align_up(w.part_ml + bhs * kMaxNodes * sizeof(float2), 256);
+  w.total = adt::align_up(w.part_o + bhs * kMaxNodes * D * sizeof(float), 256);
   return w;
 }
 
@@ -431,7 +436,7 @@ extern "C" {
 size_t adt_tree_attn_workspace_size(int32_t B, int32_t H, int32_t D, int32_t max_nodes,
                                     int32_t max_kv) {
   (void)max_nodes;
-  if (B < 1 || H < 1 || (D != 64 && D != 128) || max_kv < 0) return 0;
+  if (B < 1 || H < 1 || (D != 64 && D != 128) || max_kv < 0 || static_cast<int64_t>(B) * H > kMaxBH) return 0;
   adt::DeviceInfo info;
   if (adt::device_info(&info) != ADT_OK) return 0;
   return ws_layout(B, H, D, choose_splits(info.sm_count, B, H, D, max_kv)).total;
@@ -445,6 +450,7 @@ adt_status adt_tree_attn(const adt_bf16* q, const adt_bf16* k_cache, const adt_b
                          float* lse, void* workspace, size_t workspace_bytes, void* stream) {
   ADT_REQUIRE(q && k_cache && v_cache && kv_len && k_tree && v_tree && parents && node_offsets && out);
   ADT_REQUIRE(B >= 1 && H >= 1 && Hkv >= 1 && H % Hkv == 0);
+  ADT_REQUIRE(static_cast<int64_t>(B) * H <= kMaxBH && B <= 65535 && H <= 65535);
   ADT_REQUIRE(max_nodes >= 1 && max_kv >= 0);
   ADT_REQUIRE(softmax_scale > 0.f && softmax_scale < 1e30f);
   if (D != 64 && D != 128) return ADT_ERR_UNSUPPORTED;

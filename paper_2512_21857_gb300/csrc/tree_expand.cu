@@ -171,20 +171,25 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
   if (tid == 0) *p.all_ticket = 0u;
 }
 
+// Workspace layout.  The completion counters sit at fixed offsets at the
+// start (room for the largest F), so calls of any shape can share one
+// workspace; the data regions after them are rewritten before being read.
+constexpr int kMaxRows = 4096;
+
 struct ExpandWs {
-  size_t part_keys, part_max, part_sum, cross_keys, row_tickets, all_ticket, total;
+  size_t row_tickets, all_ticket, part_keys, part_max, part_sum, cross_keys, total;
 };
 
 ExpandWs expand_ws(int F, int V, int k) {
   const size_t S = (static_cast<size_t>(V) + kChunk - 1) / kChunk;
   ExpandWs w{};
-  w.part_keys = 0;
+  w.row_tickets = 0;
+  w.all_ticket = kMaxRows * sizeof(unsigned);
+  w.part_keys = adt::align_up(w.all_ticket + sizeof(unsigned), 256);
   w.part_max = adt::align_up(w.part_keys + F * S * k * sizeof(uint64_t), 256);
   w.part_sum = adt::align_up(w.part_max + F * S * sizeof(float), 256);
   w.cross_keys = adt::align_up(w.part_sum + F * S * sizeof(double), 256);
-  w.row_tickets = adt::align_up(w.cross_keys + static_cast<size_t>(F) * k * sizeof(uint64_t), 256);
-  w.all_ticket = adt::align_up(w.row_tickets + F * sizeof(unsigned), 256);
-  w.total = adt::align_up(w.all_ticket + sizeof(unsigned), 256);
+  w.total = adt::align_up(w.cross_keys + static_cast<size_t>(F) * k * sizeof(uint64_t), 256);
   return w;
 }
 
@@ -308,7 +313,7 @@ adt_status adt_tree_expand(const float* logits, int64_t ld, const float* frontie
                            int32_t* next_id, void* workspace, size_t workspace_bytes,
                            void* stream) {
   ADT_REQUIRE(logits && frontier_score && child_token && child_score && child_parent && keep_idx);
-  ADT_REQUIRE(F >= 1 && F <= 4096 && V >= 1 && V <= (1 << 24));
+  ADT_REQUIRE(F >= 1 && F <= kMaxRows && V >= 1 && V <= (1 << 24));
   ADT_REQUIRE(k_child >= 1 && k_child <= kMaxK && k_child <= V);
   ADT_REQUIRE(k_keep >= 1 && k_keep <= F * k_child && k_keep <= kMaxKeep);
   ADT_REQUIRE(ld >= V && ld % 4 == 0 && adt::aligned16(logits));

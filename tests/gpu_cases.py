@@ -47,13 +47,14 @@ class AttnCase:
         self.vt = synth.bf16_normal((ntot, Hkv, D), seed, "vt")
         self.scale = 1.0 / math.sqrt(D)
 
-    def run_gpu(self, max_nodes=None, max_kv=None):
+    def run_gpu(self, max_nodes=None, max_kv=None, ws=None):
         dev = "cuda"
         max_nodes = max_nodes or max(self.sizes)
         max_kv = max(self.kv_lens) if max_kv is None else max_kv
         out = torch.empty((self.ntot, self.H, self.D), dtype=torch.bfloat16, device=dev)
         lse = torch.empty((self.ntot, self.H), dtype=torch.float32, device=dev)
-        ws = B.zeroed_workspace(B.adt_tree_attn_workspace_size(self.B, self.H, self.D, max_nodes, max_kv))
+        if ws is None:
+            ws = B.zeroed_workspace(B.adt_tree_attn_workspace_size(self.B, self.H, self.D, max_nodes, max_kv))
         kc, vc = self.kc.to(dev), self.vc.to(dev)
         B.adt_tree_attn(self.q.to(dev), kc, vc, i32(self.kv_lens), self.kt.to(dev), self.vt.to(dev),
                         i32(self.tb.parents), i32(self.tb.node_offsets), B=self.B, H=self.H, Hkv=self.Hkv, D=self.D,

@@ -22,10 +22,11 @@ def _built():
     ensure_built()
 
 
-def run_expand(logits, fscore, fid, k, keep, T=1.0, base=0):
+def run_expand(logits, fscore, fid, k, keep, T=1.0, base=0, ws=None):
     F, V = logits.shape
     dev = "cuda"
-    ws = B.zeroed_workspace(B.adt_tree_expand_workspace_size(F, V, k))
+    if ws is None:
+        ws = B.zeroed_workspace(B.adt_tree_expand_workspace_size(F, V, k))
     out = dict(child_token=torch.empty(F * k, dtype=torch.int32, device=dev),
                child_logp=torch.empty(F * k, dtype=torch.float32, device=dev),
                child_score=torch.empty(F * k, dtype=torch.float32, device=dev),
@@ -33,14 +34,17 @@ def run_expand(logits, fscore, fid, k, keep, T=1.0, base=0):
     keep_idx = torch.empty(keep, dtype=torch.int32, device=dev)
     ns = torch.empty(keep, dtype=torch.float32, device=dev)
     nid = torch.empty(keep, dtype=torch.int32, device=dev)
-    B.adt_tree_expand(f32(logits), f32(fscore), None if fid is None else i32(fid), F=F, V=V, k_child=k,
+    ld = (V + 3) // 4 * 4  # rows padded to a multiple of 4 floats, as the ABI requires
+    padded = torch.zeros((F, ld), dtype=torch.float32, device=dev)
+    padded[:, :V] = f32(logits)
+    B.adt_tree_expand(padded[:, :V], f32(fscore), None if fid is None else i32(fid), F=F, V=V, k_child=k,
                       k_keep=keep, temperature=T, child_id_base=base, keep_idx=keep_idx, next_score=ns,
                       next_id=nid, workspace=ws, **out)
     torch.cuda.synchronize()
     res = {kk: v.cpu().numpy() for kk, v in out.items()}
     res.update(keep_idx=keep_idx.cpu().numpy(), next_score=ns.cpu().numpy(), next_id=nid.cpu().numpy())
-    # the completion counters (end of the workspace) are back at zero
-    assert int(ws[-256:].cpu().sum()) == 0
+    # the completion counters (start of the workspace) are back at zero
+    assert int(ws[:16640].cpu().sum()) == 0
     return res, ws
 
 
@@ -97,13 +101,20 @@ def test_expand_ties_take_lowest_index():
     check_expand(got, ref, 5)
 
 
-def test_expand_repeated_calls_reuse_workspace():
-    logits = synth.f32_normal((8, 65536), 9, "l")
-    fs = np.zeros(8, np.float32)
-    a, _ = run_expand(logits, fs, None, 8, 8)
-    b, _ = run_expand(logits, fs, None, 8, 8)
-    for key in a:
-        assert np.array_equal(a[key], b[key])
+def test_expand_shared_workspace_across_shapes_and_repeats():
+    """One workspace serves calls of different F in any order (a step's
+    first layer has F = 1, later ones F = k), repeatedly."""
+    V = 65536
+    ws = B.zeroed_workspace(B.adt_tree_expand_workspace_size(8, V, 8))
+    rows1 = synth.f32_normal((1, V), 11, "a")
+    rows8 = synth.f32_normal((8, V), 11, "b")
+    ref1 = oracle.tree_expand(rows1, np.zeros(1, np.float32), 8, 8)
+    ref8 = oracle.tree_expand(rows8, np.zeros(8, np.float32), 8, 8)
+    for _ in range(3):
+        g1, _ = run_expand(rows1, np.zeros(1, np.float32), None, 8, 8, ws=ws)
+        check_expand(g1, ref1, 8)
+        g8, _ = run_expand(rows8, np.zeros(8, np.float32), None, 8, 8, ws=ws)
+        check_expand(g8, ref8, 8)
 
 
 def _oracle_grow(draft_rows, k, depth, root_token, n_nodes):
