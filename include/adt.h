@@ -139,6 +139,36 @@ adt_status adt_tree_attn(const adt_bf16* q, const adt_bf16* k_cache, const adt_b
                          float* lse, void* workspace, size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
+ * adt_tree_attn_noalloc - adt_tree_attn without a workspace argument.
+ *
+ * The paper has no counterpart: this entry point exists for callers that
+ * cannot allocate device memory themselves (a plugin whose host engine owns
+ * every device allocation; a latency-critical thread that must not call
+ * cudaMalloc, which may synchronise the device).  It computes what
+ * adt_tree_attn computes, with the same arguments minus the workspace, and
+ * allocates nothing: its scratch is one fixed 8 MiB array per device, held
+ * by every GPU that loads the library until the process exits.
+ *   - The first call on each device looks up that array's device address;
+ *     make this first call before any stream capture begins.
+ *   - Every call shares the array (it keeps the last call's contents; the
+ *     call clears what must start at zero on `stream` itself).  Calls that
+ *     overlap on the GPU (other streams, other host threads) race on it:
+ *     serialise them.
+ *   - The key range is split into fewer pieces when the partial results of
+ *     the usual split would not fit; a shape whose partials do not fit even
+ *     unsplit (B * H * 64 * (D + 2) * 4 bytes plus tickets > 8 MiB) returns
+ *     ADT_ERR_WORKSPACE and launches nothing.
+ * ------------------------------------------------------------------------ */
+adt_status adt_tree_attn_noalloc(const adt_bf16* q, const adt_bf16* k_cache,
+                                 const adt_bf16* v_cache, const int32_t* kv_len,
+                                 int64_t cache_stride_b, int64_t cache_stride_h,
+                                 const adt_bf16* k_tree, const adt_bf16* v_tree,
+                                 const int32_t* parents, const int32_t* node_offsets, int32_t B,
+                                 int32_t H, int32_t Hkv, int32_t D, int32_t max_nodes,
+                                 int32_t max_kv, float softmax_scale, adt_bf16* out, float* lse,
+                                 void* stream);
+
+/* ------------------------------------------------------------------------
  * adt_tree_expand - one layer of dynamic draft-tree growth (Sec. 3.1 last
  * paragraph; Sec. 4.2 / Fig. 5; node score Eq. 4 in the log domain).
  *

@@ -25,7 +25,7 @@ DEVERR_BAD_TREE, DEVERR_KV_RANGE, DEVERR_BAD_PATH, DEVERR_TIMEOUT, DEVERR_BAD_IN
 
 EXPORTED = [
     "adt_version", "adt_get_device_error", "adt_status_string",
-    "adt_tree_attn_workspace_size", "adt_tree_attn",
+    "adt_tree_attn_workspace_size", "adt_tree_attn", "adt_tree_attn_noalloc",
     "adt_tree_expand_workspace_size", "adt_tree_expand",
     "adt_tree_rerank_workspace_size", "adt_tree_rerank",
     "adt_tree_accept_workspace_size", "adt_tree_accept",
@@ -56,6 +56,8 @@ _SIGS = {
     "adt_tree_attn_workspace_size": ([_I32] * 5, _SZ),
     "adt_tree_attn": ([_P, _P, _P, _P, _I64, _I64, _P, _P, _P, _P, _I32, _I32, _I32, _I32, _I32, _I32, _F32,
                        _P, _P, _P, _SZ, _P], _I32),
+    "adt_tree_attn_noalloc": ([_P, _P, _P, _P, _I64, _I64, _P, _P, _P, _P, _I32, _I32, _I32, _I32, _I32, _I32,
+                               _F32, _P, _P, _P], _I32),
     "adt_tree_expand_workspace_size": ([_I32] * 3, _SZ),
     "adt_tree_expand": ([_P, _I64, _P, _P, _I32, _I32, _I32, _I32, _F32, _I32, _P, _P, _P, _P, _P, _P, _P,
                          _P, _SZ, _P], _I32),

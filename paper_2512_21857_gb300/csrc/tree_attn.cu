@@ -495,3 +495,114 @@ adt_status adt_tree_attn(const adt_bf16* q, const adt_bf16* k_cache, const adt_b
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// adt_tree_attn_noalloc: the same tree attention for callers that cannot
+// allocate device memory themselves, for example a plugin inside a serving
+// engine whose host owns every device allocation, or code on a latency-
+// critical thread that must not call cudaMalloc (it can synchronise the
+// device).  The split partials and completion tickets live in one fixed,
+// per-device static array instead of a caller-provided workspace.
+// ---------------------------------------------------------------------------
+
+#include <mutex>
+
+// 8 MiB of scratch, held by every GPU that loads the library until the
+// process exits.  Shared by all calls on a device: calls that overlap on the
+// GPU (different streams, or different host threads) race on it.
+static constexpr size_t kNoAllocScratchBytes = size_t(8) << 20;
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+namespace {
+
+constexpr int kNoAllocMaxDevices = 64;
+std::once_flag g_noalloc_once[kNoAllocMaxDevices];
+void* g_noalloc_ptr[kNoAllocMaxDevices];
+cudaError_t g_noalloc_status[kNoAllocMaxDevices];
+
+// Runs once per device, with that device current: the array's name is a
+// host-side stand-in in host code, so the kernel needs its device address.
+void noalloc_setup(int dev) {
+  void* p = nullptr;
+  g_noalloc_status[dev] = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+  g_noalloc_ptr[dev] = p;
+}
+
+struct NoAllocLayout {
+  size_t tickets, part_ml, part_o, total;
+};
+
+NoAllocLayout noalloc_layout(int B, int H, int D, int splits) {
+  NoAllocLayout w{};
+  const size_t bh = static_cast<size_t>(B) * H;
+  const size_t bhs = bh * splits;
+  w.tickets = 0;
+  w.part_ml = adt::align_up(bh * sizeof(unsigned), 256);
+  w.part_o = adt::align_up(w.part_ml + bhs * kMaxNodes * sizeof(float2), 256);
+  w.total = adt::align_up(w.part_o + bhs * kMaxNodes * D * sizeof(float), 256);
+  return w;
+}
+
+}  // namespace
+
+extern "C" adt_status adt_tree_attn_noalloc(const adt_bf16* q, const adt_bf16* k_cache,
+                                            const adt_bf16* v_cache, const int32_t* kv_len,
+                                            int64_t cache_stride_b, int64_t cache_stride_h,
+                                            const adt_bf16* k_tree, const adt_bf16* v_tree,
+                                            const int32_t* parents, const int32_t* node_offsets,
+                                            int32_t B, int32_t H, int32_t Hkv, int32_t D,
+                                            int32_t max_nodes, int32_t max_kv, float softmax_scale,
+                                            adt_bf16* out, float* lse, void* stream) {
+  ADT_REQUIRE(q && k_cache && v_cache && kv_len && k_tree && v_tree && parents && node_offsets && out);
+  ADT_REQUIRE(B >= 1 && H >= 1 && Hkv >= 1 && H % Hkv == 0);
+  ADT_REQUIRE(B <= 65535 && H <= 65535);
+  ADT_REQUIRE(max_nodes >= 1 && max_kv >= 0);
+  ADT_REQUIRE(softmax_scale > 0.f && softmax_scale < 1e30f);
+  if (D != 64 && D != 128) return ADT_ERR_UNSUPPORTED;
+  if (max_nodes > kMaxNodes) return ADT_ERR_UNSUPPORTED;
+  ADT_REQUIRE(cache_stride_b >= 0 && cache_stride_h >= 0 && cache_stride_b % 8 == 0 &&
+              cache_stride_h % 8 == 0);
+  ADT_REQUIRE(adt::aligned16(q) && adt::aligned16(k_cache) && adt::aligned16(v_cache) &&
+              adt::aligned16(k_tree) && adt::aligned16(v_tree) && adt::aligned16(out));
+  adt::DeviceInfo info;
+  adt_status st = adt::device_info(&info);
+  if (st != ADT_OK) return st;
+  if (info.device < 0 || info.device >= kNoAllocMaxDevices) return ADT_ERR_UNSUPPORTED;
+  std::call_once(g_noalloc_once[info.device], noalloc_setup, info.device);
+  if (g_noalloc_status[info.device] != cudaSuccess || !g_noalloc_ptr[info.device]) return ADT_ERR_CUDA;
+  // As many splits as the usual heuristic picks, fewer if the partials would
+  // not fit; a shape that does not fit even unsplit is rejected.
+  int splits = choose_splits(info.sm_count, B, H, D, max_kv);
+  while (splits > 1 && noalloc_layout(B, H, D, splits).total > kNoAllocScratchBytes) --splits;
+  const NoAllocLayout w = noalloc_layout(B, H, D, splits);
+  if (w.total > kNoAllocScratchBytes) return ADT_ERR_WORKSPACE;
+  uint8_t* ws = static_cast<uint8_t*>(g_noalloc_ptr[info.device]);
+  cudaStream_t s = adt::as_stream(stream);
+  // The array keeps the previous call's contents: the tickets must start at zero.
+  ADT_CUDA_TRY(cudaMemsetAsync(ws + w.tickets, 0, static_cast<size_t>(B) * H * sizeof(unsigned), s));
+  AttnParams prm;
+  prm.q = reinterpret_cast<const __nv_bfloat16*>(q);
+  prm.kc = reinterpret_cast<const __nv_bfloat16*>(k_cache);
+  prm.vc = reinterpret_cast<const __nv_bfloat16*>(v_cache);
+  prm.kv_len = kv_len;
+  prm.sb = cache_stride_b;
+  prm.sh = cache_stride_h;
+  prm.kt = reinterpret_cast<const __nv_bfloat16*>(k_tree);
+  prm.vt = reinterpret_cast<const __nv_bfloat16*>(v_tree);
+  prm.parents = parents;
+  prm.offs = node_offsets;
+  prm.B = B;
+  prm.H = H;
+  prm.Hkv = Hkv;
+  prm.group = H / Hkv;
+  prm.max_kv = max_kv;
+  prm.splits = splits;
+  prm.scale_log2 = softmax_scale * kLog2e;
+  prm.out = reinterpret_cast<__nv_bfloat16*>(out);
+  prm.lse = lse;
+  prm.part_o = reinterpret_cast<float*>(ws + w.part_o);
+  prm.part_ml = reinterpret_cast<float2*>(ws + w.part_ml);
+  prm.tickets = reinterpret_cast<unsigned*>(ws + w.tickets);
+  prm.err = info.error_word;
+  return D == 128 ? launch<128>(prm, s, info.device) : launch<64>(prm, s, info.device);
+}
