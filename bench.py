@@ -418,7 +418,7 @@ def main():
         "warmup": args.warmup, "ms_per_step": r["step_ms"], "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config,
         "hbm_gbs_step": r["step_bytes"] / (r["step_ms"] * 1e-3) / 1e9,
-        "roofline": {"bound": "hbm", "kernel": "tree_attn_kernel<128>" if wl["D"] == 128 else "tree_attn_kernel<64>",
+        "roofline": {"bound": "hbm", "kernel": "tree_attn_tc_kernel<128>" if wl["D"] == 128 else "tree_attn_tc_kernel<64>",
                      "achieved": r["achieved"], "peak": r["peak"], "unit": "GB/s",
                      "frac": r["achieved"] / r["peak"], "peak_source": f"{r['peak_kind']} (hbm_gbs)",
                      "traffic": r["traffic"], "algorithmic_bytes_per_launch": r["attn_bytes"],

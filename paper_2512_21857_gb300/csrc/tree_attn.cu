@@ -3,129 +3,166 @@
 // conditioned on s_{1:t} and ans(t) under the tree mask; the mask is the
 // T_N term of Eq. 5).
 //
-// Split-KV flash decoding.  The keys a tree sees are cut into units of 64:
-// ceil(L/64) prefix units plus one tree unit (the <= 64 tree nodes, masked
-// per row by an ancestor bitmask built from the parent pointers).  Grid =
-// (splits, H, B); a CTA streams its share of units for one (tree, head)
-// through a 3-stage cp.async pipeline into XOR-swizzled shared memory and
-// runs QK^T and PV on bf16 mma.sync tiles (m16n8k16, fp32 accumulation) with
-// an online softmax in registers.  Each warp owns 16 query rows.  The CTA
-// that finishes a (tree, head) last (atomic ticket) merges the split
-// partials (m, l, unnormalised O) and writes bf16 O and the natural-log LSE.
+// Split-KV flash decoding on the 5th-generation tensor cores.  The keys a
+// tree sees are cut into units of 64: ceil(L/64) prefix units plus one tree
+// unit (its <= 64 nodes, masked per query row by an ancestor bitmask built
+// from the parent pointers).  Grid = (splits, H, B), one CTA per SM; a CTA
+// handles one (tree, head) and a contiguous share of the units.
+//
+// Warp roles inside a CTA (192 threads):
+//   warp 4    producer: TMA tensor loads of prefix K/V chunks (128-byte
+//             swizzle) into a ring of stages; the tree unit (rows of
+//             k_tree / v_tree that TMA cannot bound) with cp.async;
+//   warp 5    one elected thread issues tcgen05.mma: S = Q K^T into a
+//             double-buffered tensor-memory tile (M = 64 queries, N = 64
+//             keys), then O += P V (N = head_dim, V read MN-major);
+//   warps 0-3 softmax: each thread owns one query row (tensor-memory lane
+//             32w + i holds row 16w + i for M = 64), reads its S row,
+//             masks, exponentiates with a lazily raised running maximum
+//             (O is rescaled only when the maximum grows by more than 2^8),
+//             writes P (bf16) to shared memory for the PV product; at the
+//             end they read O and l and emit the split's partial.
+// mbarriers connect the roles; every wait is bounded and a timeout sets
+// ADT_DEVERR_TIMEOUT.  The splits of one (tree, head) form a thread-block
+// cluster (<= 8) and merge their partials through distributed shared
+// memory; with more splits they merge through the workspace.
+#include <cooperative_groups.h>
+#include <cuda.h>
+
+#include <mutex>
+
 #include "adt_common.cuh"
+#include "sm100.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace {
 
-constexpr int kKeys = 64;
-constexpr int kStages = 3;
-constexpr int kWarps = 4;
-constexpr int kThreads = kWarps * 32;
-constexpr int kMaxNodes = 64;
+constexpr int kUnit = 64;               // keys per pipeline unit
+constexpr int kMaxNodes = 64;           // tree nodes (query rows) per (tree, head)
+constexpr int kSoftmaxWarps = 4;
+constexpr int kProducerWarp = 4;
+constexpr int kMmaWarp = 5;
+constexpr int kThreads = 6 * 32;
+constexpr int kMaxClusterSplits = 8;    // portable cluster size
+constexpr int kMaxSplits = 96;          // workspace merge: weights fit in shared memory
+constexpr int kMaxStages = 8;
+constexpr uint32_t kWaitLimit = 1u << 20;
+constexpr uint32_t kTmemCols = 256;     // S double buffer (2 x 64 columns) + O (<= 128 columns)
+constexpr uint32_t kOCol = 128;
 constexpr float kLn2 = 0.69314718055994530942f;
 constexpr float kLog2e = 1.44269504088896340736f;
+constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 template <int D>
 struct Cfg {
-  static constexpr int kRowBytes = D * 2;
-  static constexpr int kChunks = kRowBytes / 16;  // 16-byte chunks per key row
-  static constexpr int kTileBytes = kKeys * kRowBytes;
-  static constexpr int kStageBytes = 2 * kTileBytes;  // K tile + V tile
-  static constexpr int kSmemBytes = kStages * kStageBytes + kMaxNodes * 8;
-  static constexpr int kKSteps = D / 16;  // k-steps of QK^T
-  static constexpr int kNTiles = D / 8;   // n-tiles of O
+  static constexpr int kBlocks = D / 64;             // 128-byte column blocks per row
+  static constexpr int kBlockBytes = kUnit * 128;    // one column block of 64 rows
+  static constexpr int kTileBytes = kBlocks * kBlockBytes;  // 64 rows x D bf16
+  static constexpr int kStages = D == 128 ? 5 : 8;
+  static constexpr int kQOff = 0;
+  static constexpr int kPOff = kTileBytes;                  // two P buffers (64 x 64 bf16)
+  static constexpr int kTrashOff = kPOff + 2 * kBlockBytes; // 16 scratch rows for idle lanes
+  static constexpr int kStageOff = kTrashOff + 2048;
+  static constexpr int kStageBytes = 2 * kTileBytes;        // K tile, then V tile
+  static constexpr int kDynSmem = kStageOff + kStages * kStageBytes + 1024;  // + alignment slack
+  static constexpr uint32_t kIdescS = sm100::idesc_bf16_f32(64, 64, 0, 0);
+  static constexpr uint32_t kIdescO = sm100::idesc_bf16_f32(64, D, 0, 1);
+  static constexpr int kMergeStride = D + 4;                // fp32 per row of a parked partial
 };
 
-struct AttnParams {
+struct TcParams {
   const __nv_bfloat16* q;
-  const __nv_bfloat16* kc;
-  const __nv_bfloat16* vc;
-  const int32_t* kv_len;
-  int64_t sb, sh;
   const __nv_bfloat16* kt;
   const __nv_bfloat16* vt;
+  const int32_t* kv_len;
   const int32_t* parents;
   const int32_t* offs;
   int B, H, Hkv, group, max_kv, splits;
+  int cluster_merge;
   float scale_log2;
   __nv_bfloat16* out;
   float* lse;
-  float* part_o;   // [B][H][splits][64][D]
-  float2* part_ml; // [B][H][splits][64]
+  float* part_o;      // [B][H][splits][64][D]   (workspace merge only)
+  float2* part_ml;    // [B][H][splits][64]
   unsigned* tickets;  // [B][H]
   unsigned* err;
 };
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+// Byte offset of 16-byte chunk `ch` (0 .. D/8-1) of row `row` in a tile of
+// 128-byte column blocks with the 128-byte swizzle (the layout TMA writes).
+__device__ __forceinline__ uint32_t sw128_off(int row, int ch) {
+  return static_cast<uint32_t>((ch >> 3) * (kUnit * 128) + row * 128 + (((ch & 7) ^ (row & 7)) << 4));
 }
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes));
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
 }
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;\n" ::"n"(N));
-}
-
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
-                                        uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-__device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t& r0, uint32_t& r1,
-                                              uint32_t& r2, uint32_t& r3) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
-               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-               : "r"(addr));
-}
-
-__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
-                                               uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-      "{%8,%9}, {%0,%1,%2,%3};\n"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;\n" ::: "memory"); }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// Byte offset of 16-byte chunk `ch` of key row `row` inside a swizzled tile.
-template <int D>
-__device__ __forceinline__ uint32_t tile_off(int row, int ch) {
-  return static_cast<uint32_t>(row * Cfg<D>::kRowBytes + ((ch ^ (row & 7)) << 4));
+struct Barriers {
+  uint64_t q_full;
+  uint64_t kv_full[kMaxStages];
+  uint64_t kv_empty[kMaxStages];
+  uint64_t s_full[2];
+  uint64_t s_free[2];
+  uint64_t p_full[2];
+  uint64_t pv_done[2];
+  uint64_t o_full;
+};
+
+// Bounded wait that also gives up when another role has aborted.
+__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                         unsigned* err) {
+  const uint32_t a = sm100::smem_addr(bar);
+  for (uint32_t i = 0; i < kWaitLimit; ++i) {
+    if (sm100::mbar_try_wait(a, parity)) return true;
+    if ((i & 255u) == 255u && *abort_flag) return false;
+  }
+  *abort_flag = 1;
+  adt::raise_error(err, ADT_DEVERR_TIMEOUT);
+  return false;
 }
 
 template <int D>
-__global__ void __launch_bounds__(kThreads) tree_attn_kernel(const AttnParams p) {
+__global__ void __launch_bounds__(kThreads, 1)
+    tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+                        const TcParams p) {
   using C = Cfg<D>;
-  extern __shared__ __align__(128) uint8_t smem[];
-  uint64_t* anc = reinterpret_cast<uint64_t*>(smem + kStages * C::kStageBytes);
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  __shared__ Barriers bars;
+  __shared__ uint64_t anc[kMaxNodes];
+  __shared__ uint32_t tmem_slot;
   __shared__ int s_bad;
   __shared__ int s_last;
+  __shared__ volatile int s_abort;
 
   const int split = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int g = h / p.group;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int grp = lane >> 2, tig = lane & 3;
 
   const int node0 = p.offs[b];
   const int n = p.offs[b + 1] - node0;
   const int L = p.kv_len[b];
 
-  if (tid == 0) s_bad = 0;
+  if (tid == 0) {
+    s_bad = 0;
+    s_abort = 0;
+  }
   __syncthreads();
+  // Conditions that hold for every CTA of this (tree, head): all leave here.
   if (n < 1 || n > kMaxNodes) {
-    if (split == 0 && h == 0) adt::raise_error(p.err, ADT_DEVERR_BAD_TREE);
-    return;  // uniform over the CTA and over every split of this (b, h)
+    if (split == 0 && h == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_BAD_TREE);
+    return;
   }
   if (L < 0 || L > p.max_kv) {
-    if (split == 0 && h == 0) adt::raise_error(p.err, ADT_DEVERR_KV_RANGE);
+    if (split == 0 && h == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_KV_RANGE);
     return;
   }
   // Ancestor bitmask of every node: bit j of anc[t] <=> j in ans(t) or j == t.
@@ -154,244 +191,431 @@ __global__ void __launch_bounds__(kThreads) tree_attn_kernel(const AttnParams p)
   }
   __syncthreads();
   if (s_bad) {
-    if (split == 0 && h == 0) adt::raise_error(p.err, ADT_DEVERR_BAD_TREE);
+    if (split == 0 && h == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_BAD_TREE);
     return;
   }
 
-  const int U = (L + kKeys - 1) / kKeys + 1;  // prefix units + the tree unit
+  const int U = (L + kUnit - 1) / kUnit + 1;  // prefix units + the tree unit
   const int S = p.splits;
   const int u_begin = static_cast<int>(static_cast<int64_t>(split) * U / S);
   const int u_end = static_cast<int>(static_cast<int64_t>(split + 1) * U / S);
   const int nu = u_end - u_begin;
+  const int NS = C::kStages;
 
-  const __nv_bfloat16* kc_bh = p.kc + b * p.sb + g * p.sh;
-  const __nv_bfloat16* vc_bh = p.vc + b * p.sb + g * p.sh;
+  uint8_t* sQ = smem + C::kQOff;
+  uint8_t* sP = smem + C::kPOff;
+  uint8_t* sStage = smem + C::kStageOff;
+  uint8_t* sTrash = smem + C::kTrashOff;
 
-  auto load_unit = [&](int u, int stage) {
-    const uint32_t ks = smem_u32(smem + stage * C::kStageBytes);
-    const bool tree = (u == U - 1);
-    for (int i = tid; i < kKeys * C::kChunks; i += kThreads) {
-      const int row = i / C::kChunks, ch = i % C::kChunks;
-      const __nv_bfloat16* ksrc;
-      const __nv_bfloat16* vsrc;
-      bool valid;
-      if (!tree) {
-        const int key = u * kKeys + row;
-        valid = key < L;
-        const int64_t off = static_cast<int64_t>(valid ? key : 0) * D + ch * 8;
-        ksrc = kc_bh + off;
-        vsrc = vc_bh + off;
-      } else {
-        valid = row < n;
-        const int64_t off = (static_cast<int64_t>(node0 + (valid ? row : 0)) * p.Hkv + g) * D + ch * 8;
-        ksrc = p.kt + off;
-        vsrc = p.vt + off;
-      }
-      const uint32_t dst = ks + tile_off<D>(row, ch);
-      cp_async16(dst, ksrc, valid ? 16 : 0);
-      cp_async16(dst + C::kTileBytes, vsrc, valid ? 16 : 0);
+  if (tid == 0) {
+    sm100::mbar_init(sm100::smem_addr(&bars.q_full), kSoftmaxWarps);
+    for (int s = 0; s < NS; ++s) {
+      sm100::mbar_init(sm100::smem_addr(&bars.kv_full[s]), 1);
+      sm100::mbar_init(sm100::smem_addr(&bars.kv_empty[s]), 1);
     }
-  };
-
-  // Query fragments (A operand of QK^T) for rows r0 = 16*warp + grp and r0 + 8.
-  const int r0 = warp * 16 + grp, r1 = r0 + 8;
-  const bool warp_active = warp * 16 < n;
-  uint32_t qa[C::kKSteps][4];
-  {
-    const __nv_bfloat16* q0 = p.q + (static_cast<int64_t>(node0 + r0) * p.H + h) * D;
-    const __nv_bfloat16* q1 = p.q + (static_cast<int64_t>(node0 + r1) * p.H + h) * D;
-#pragma unroll
-    for (int kk = 0; kk < C::kKSteps; ++kk) {
-      const int d0 = kk * 16 + tig * 2;
-      qa[kk][0] = r0 < n ? *reinterpret_cast<const uint32_t*>(q0 + d0) : 0u;
-      qa[kk][1] = r1 < n ? *reinterpret_cast<const uint32_t*>(q1 + d0) : 0u;
-      qa[kk][2] = r0 < n ? *reinterpret_cast<const uint32_t*>(q0 + d0 + 8) : 0u;
-      qa[kk][3] = r1 < n ? *reinterpret_cast<const uint32_t*>(q1 + d0 + 8) : 0u;
+    for (int s = 0; s < 2; ++s) {
+      sm100::mbar_init(sm100::smem_addr(&bars.s_full[s]), 1);
+      sm100::mbar_init(sm100::smem_addr(&bars.s_free[s]), kSoftmaxWarps);
+      sm100::mbar_init(sm100::smem_addr(&bars.p_full[s]), kSoftmaxWarps);
+      sm100::mbar_init(sm100::smem_addr(&bars.pv_done[s]), 1);
     }
+    sm100::mbar_init(sm100::smem_addr(&bars.o_full), 1);
+    sm100::fence_mbar_init();
   }
-
-  float o[C::kNTiles][4];
-#pragma unroll
-  for (int t = 0; t < C::kNTiles; ++t) o[t][0] = o[t][1] = o[t][2] = o[t][3] = 0.f;
-  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
-  const uint64_t anc0 = r0 < n ? anc[r0] : 0ull;
-  const uint64_t anc1 = r1 < n ? anc[r1] : 0ull;
-
-#pragma unroll
-  for (int s = 0; s < kStages - 1; ++s) {
-    if (s < nu) load_unit(u_begin + s, s);
-    cp_async_commit();
+  if (warp == 0) {
+    sm100::tmem_alloc(sm100::smem_addr(&tmem_slot), kTmemCols);
+    sm100::tmem_relinquish();
   }
+  sm100::tc_fence_before();
+  __syncthreads();
+  sm100::tc_fence_after();
+  const uint32_t tmem = tmem_slot;
 
-  for (int it = 0; it < nu; ++it) {
-    cp_async_wait<kStages - 2>();
-    __syncthreads();
-    {
-      const int nx = it + kStages - 1;
-      if (nx < nu) load_unit(u_begin + nx, nx % kStages);
-      cp_async_commit();
-    }
-    if (!warp_active) continue;
-    const int u = u_begin + it;
-    const uint32_t ks = smem_u32(smem + (it % kStages) * C::kStageBytes);
-    const uint32_t vs = ks + C::kTileBytes;
-    const bool tree = (u == U - 1);
+  // Per-row state of the softmax threads (lane < 16 of warps 0-3).
+  const int row = warp * 16 + lane;
+  float m_used = -INFINITY, l_sum = 0.f;
 
-    float s[8][4];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
-    const int mat = lane >> 3, mr = lane & 7;
-#pragma unroll
-    for (int kk = 0; kk < C::kKSteps; ++kk) {
-#pragma unroll
-      for (int j = 0; j < 8; j += 2) {
-        const int row = (j + (mat >> 1)) * 8 + mr;
-        const int ch = 2 * kk + (mat & 1);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(ks + tile_off<D>(row, ch), b0, b1, b2, b3);
-        mma_bf16_16816(s[j], qa[kk], b0, b1);
-        mma_bf16_16816(s[j + 1], qa[kk], b2, b3);
-      }
-    }
-    // Mask, scale to the log2 domain, online softmax.
-    float mx0 = -INFINITY, mx1 = -INFINITY;
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int key = j * 8 + tig * 2 + (e & 1);
-        bool ok;
-        if (tree) {
-          ok = ((e < 2 ? anc0 : anc1) >> key) & 1ull;
-        } else {
-          ok = u * kKeys + key < L;
+  if (warp == kProducerWarp) {
+    // ------------------------------------------------------------ producer
+    int issued = 0;
+    for (int j = 0; j < nu; ++j) {
+      const int st = j % NS;
+      if (j >= NS &&
+          !__all_sync(adt::kFullMask, wait_bar(&bars.kv_empty[st], ((j / NS) - 1) & 1, &s_abort, p.err)))
+        break;
+      uint8_t* kdst = sStage + st * C::kStageBytes;
+      uint8_t* vdst = kdst + C::kTileBytes;
+      const int u = u_begin + j;
+      if (u == U - 1) {
+        // Tree unit: rows node0 .. node0+63 of k_tree / v_tree for kv head g;
+        // rows past this tree are zero-filled, never read out of bounds.
+        for (int i = lane; i < kUnit * (D / 8); i += 32) {
+          const int r = i / (D / 8), ch = i % (D / 8);
+          const bool valid = r < n;
+          const int64_t off = (static_cast<int64_t>(node0 + (valid ? r : 0)) * p.Hkv + g) * D + ch * 8;
+          cp_async16(sm100::smem_addr(kdst) + sw128_off(r, ch), p.kt + off, valid ? 16 : 0);
+          cp_async16(sm100::smem_addr(vdst) + sw128_off(r, ch), p.vt + off, valid ? 16 : 0);
         }
-        const float v = ok ? s[j][e] * p.scale_log2 : -INFINITY;
-        s[j][e] = v;
-        if (e < 2) mx0 = fmaxf(mx0, v); else mx1 = fmaxf(mx1, v);
+        cp_async_wait_all();
+        sm100::fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.kv_full[st]));
+      } else if (lane == 0) {
+        const uint32_t bar = sm100::smem_addr(&bars.kv_full[st]);
+        sm100::mbar_arrive_expect_tx(bar, 2 * C::kTileBytes);
+        const int key0 = u * kUnit;
+        for (int blk = 0; blk < C::kBlocks; ++blk) {
+          sm100::tma_load_4d(sm100::smem_addr(kdst + blk * C::kBlockBytes), &tm_k, blk * 64, key0, g, b, bar);
+          sm100::tma_load_4d(sm100::smem_addr(vdst + blk * C::kBlockBytes), &tm_v, blk * 64, key0, g, b, bar);
+        }
+      }
+      __syncwarp();
+      ++issued;
+    }
+    if (s_abort && lane == 0) {
+      // let every copy still in flight land before the CTA can exit
+      for (int j = (issued > NS ? issued - NS : 0); j < issued; ++j)
+        (void)sm100::mbar_wait_bounded(sm100::smem_addr(&bars.kv_full[j % NS]), (j / NS) & 1, kWaitLimit);
+    }
+  } else if (warp == kMmaWarp) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      bool ok = wait_bar(&bars.q_full, 0, &s_abort, p.err);
+      const uint32_t q_addr = sm100::smem_addr(sQ);
+      const uint32_t p_addr = sm100::smem_addr(sP);
+      auto issue_pv = [&](int i) -> bool {
+        const int pb = i & 1;
+        if (!wait_bar(&bars.p_full[pb], (i >> 1) & 1, &s_abort, p.err)) return false;
+        sm100::tc_fence_after();
+        const uint32_t v_addr = sm100::smem_addr(sStage + (i % NS) * C::kStageBytes + C::kTileBytes);
+#pragma unroll
+        for (int kk = 0; kk < kUnit / 16; ++kk) {
+          const uint64_t da = sm100::smem_desc_sw128(p_addr + pb * C::kBlockBytes + kk * 32, 16, 1024);
+          const uint64_t db = sm100::smem_desc_sw128(v_addr + kk * 2048, C::kBlockBytes, 1024);
+          sm100::mma_bf16_ss(tmem + kOCol, da, db, C::kIdescO, (i > 0 || kk > 0) ? 1u : 0u);
+        }
+        sm100::mma_commit(sm100::smem_addr(&bars.kv_empty[i % NS]));
+        sm100::mma_commit(sm100::smem_addr(&bars.pv_done[pb]));
+        return true;
+      };
+      for (int j = 0; ok && j < nu; ++j) {
+        const int st = j % NS, sb = j & 1;
+        if (!wait_bar(&bars.kv_full[st], (j / NS) & 1, &s_abort, p.err)) break;
+        if (j >= 2 && !wait_bar(&bars.s_free[sb], ((j >> 1) - 1) & 1, &s_abort, p.err)) break;
+        sm100::tc_fence_after();
+        const uint32_t k_addr = sm100::smem_addr(sStage + st * C::kStageBytes);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * C::kBlockBytes + (kk & 3) * 32;
+          const uint64_t da = sm100::smem_desc_sw128(q_addr + off, 16, 1024);
+          const uint64_t db = sm100::smem_desc_sw128(k_addr + off, 16, 1024);
+          sm100::mma_bf16_ss(tmem + sb * 64, da, db, C::kIdescS, kk > 0 ? 1u : 0u);
+        }
+        sm100::mma_commit(sm100::smem_addr(&bars.s_full[sb]));
+        if (j >= 1 && !issue_pv(j - 1)) break;
+        if (j == nu - 1 && issue_pv(j)) sm100::mma_commit(sm100::smem_addr(&bars.o_full));
+      }
+      if (s_abort) {
+        // wait for the tensor core to finish whatever was issued
+        sm100::mma_commit(sm100::smem_addr(&bars.o_full));
+        (void)sm100::mbar_wait_bounded(sm100::smem_addr(&bars.o_full), 0, kWaitLimit);
       }
     }
-    mx0 = fmaxf(mx0, __shfl_xor_sync(adt::kFullMask, mx0, 1));
-    mx0 = fmaxf(mx0, __shfl_xor_sync(adt::kFullMask, mx0, 2));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(adt::kFullMask, mx1, 1));
-    mx1 = fmaxf(mx1, __shfl_xor_sync(adt::kFullMask, mx1, 2));
-    const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-    const float base0 = mn0 == -INFINITY ? 0.f : mn0;
-    const float base1 = mn1 == -INFINITY ? 0.f : mn1;
-    const float a0 = exp2f(m0 - base0), a1 = exp2f(m1 - base1);
-    m0 = mn0;
-    m1 = mn1;
-    float rs0 = 0.f, rs1 = 0.f;
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      s[j][0] = exp2f(s[j][0] - base0);
-      s[j][1] = exp2f(s[j][1] - base0);
-      s[j][2] = exp2f(s[j][2] - base1);
-      s[j][3] = exp2f(s[j][3] - base1);
-      rs0 += s[j][0] + s[j][1];
-      rs1 += s[j][2] + s[j][3];
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ softmax warps 0-3
+    // Q tile: rows node0 .. node0+63 (rows past the tree zero-filled).
+    for (int i = tid; i < kUnit * (D / 8); i += kSoftmaxWarps * 32) {
+      const int r = i / (D / 8), ch = i % (D / 8);
+      const bool valid = r < n;
+      const __nv_bfloat16* src = p.q + (static_cast<int64_t>(node0 + (valid ? r : 0)) * p.H + h) * D + ch * 8;
+      cp_async16(sm100::smem_addr(sQ) + sw128_off(r, ch), src, valid ? 16 : 0);
     }
-    l0 = l0 * a0 + rs0;
-    l1 = l1 * a1 + rs1;
-#pragma unroll
-    for (int t = 0; t < C::kNTiles; ++t) {
-      o[t][0] *= a0;
-      o[t][1] *= a0;
-      o[t][2] *= a1;
-      o[t][3] *= a1;
-    }
-    // O += P V
-#pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
-      uint32_t pa[4];
-      pa[0] = pack_bf16x2(s[2 * kk][0], s[2 * kk][1]);
-      pa[1] = pack_bf16x2(s[2 * kk][2], s[2 * kk][3]);
-      pa[2] = pack_bf16x2(s[2 * kk + 1][0], s[2 * kk + 1][1]);
-      pa[3] = pack_bf16x2(s[2 * kk + 1][2], s[2 * kk + 1][3]);
-#pragma unroll
-      for (int t = 0; t < C::kNTiles; t += 2) {
-        const int key = kk * 16 + (mat & 1) * 8 + mr;
-        const int ch = t + (mat >> 1);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4_trans(vs + tile_off<D>(key, ch), b0, b1, b2, b3);
-        mma_bf16_16816(o[t], pa, b0, b1);
-        mma_bf16_16816(o[t + 1], pa, b2, b3);
+    cp_async_wait_all();
+    sm100::fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.q_full));
+
+    const bool rvalid = lane < 16 && row < n;
+    const uint64_t am = rvalid ? anc[row] : 0ull;
+    const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
+    for (int j = 0; j < nu; ++j) {
+      const int sb = j & 1;
+      if (!__all_sync(adt::kFullMask, wait_bar(&bars.s_full[sb], (j >> 1) & 1, &s_abort, p.err))) break;
+      sm100::tc_fence_after();
+      const int u = u_begin + j;
+      // Which of the chunk's 64 keys this row sees: the prefix up to L, or
+      // the row's ancestors (and itself) in the tree unit.  Applied with
+      // integer bit operations so that no lane ever branches on it: the
+      // lanes of a warp hold different rows, and per-key branches would
+      // diverge.
+      uint64_t vm;
+      if (u == U - 1) {
+        vm = am;
+      } else {
+        const int kl = L - u * kUnit;  // >= 1 for every prefix unit
+        vm = kl >= 64 ? ~0ull : ((1ull << kl) - 1ull);
       }
+      const float scale = p.scale_log2;
+      const uint32_t s_addr = tmem + lane_base + sb * 64;
+      // Pass 1: row maximum of the masked, scaled scores, 16 columns at a
+      // time (the outer loops stay rolled so the hot code stays small).
+      float mx = -INFINITY;
+#pragma unroll 1
+      for (int g4 = 0; g4 < 4; ++g4) {
+        uint32_t r[16];
+        sm100::tmem_ld16(s_addr + g4 * 16, r);
+        sm100::tmem_wait_ld();
+        const uint32_t bits = static_cast<uint32_t>(vm >> (g4 * 16));
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          const uint32_t keep = 0u - ((bits >> e) & 1u);
+          const uint32_t xb = __float_as_uint(__uint_as_float(r[e]) * scale);
+          mx = fmaxf(mx, __uint_as_float((xb & keep) | (0xFF800000u & ~keep)));
+        }
+      }
+      const bool need = lane < 16 && mx > m_used + kRescaleThreshold;
+      const float new_m = need ? mx : m_used;
+      const float alpha = need ? exp2f(m_used - new_m) : 1.f;
+      const float base = new_m == -INFINITY ? 0.f : new_m;
+      // P buffer sb was last read by the PV product of chunk j - 2.
+      if (j >= 2 &&
+          !__all_sync(adt::kFullMask, wait_bar(&bars.pv_done[sb], ((j >> 1) - 1) & 1, &s_abort, p.err)))
+        break;
+      // Pass 2: p = 2^(s - base) (0 for masked keys), row sum, bf16 P row
+      // into shared memory; lanes 16-31 (no row of the M = 64 tile) write a
+      // scratch row instead of branching around the stores.
+      float rs = 0.f;
+      const uint32_t prow = lane < 16 ? sm100::smem_addr(sP + sb * C::kBlockBytes) + row * 128
+                                      : sm100::smem_addr(sTrash) + (lane - 16) * 128;
+#pragma unroll 1
+      for (int g4 = 0; g4 < 4; ++g4) {
+        uint32_t r[16];
+        sm100::tmem_ld16(s_addr + g4 * 16, r);
+        sm100::tmem_wait_ld();
+        const uint32_t bits = static_cast<uint32_t>(vm >> (g4 * 16));
+        uint32_t pk[8];
+#pragma unroll
+        for (int e = 0; e < 16; e += 2) {
+          const uint32_t k0 = 0u - ((bits >> e) & 1u), k1 = 0u - ((bits >> (e + 1)) & 1u);
+          const uint32_t x0 = __float_as_uint(__uint_as_float(r[e]) * scale);
+          const uint32_t x1 = __float_as_uint(__uint_as_float(r[e + 1]) * scale);
+          const float p0 = exp2f(__uint_as_float((x0 & k0) | (0xFF800000u & ~k0)) - base);
+          const float p1 = exp2f(__uint_as_float((x1 & k1) | (0xFF800000u & ~k1)) - base);
+          rs += p0 + p1;
+          pk[e >> 1] = pack_bf16x2(p0, p1);
+        }
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+          const int ch = g4 * 2 + h2;
+          const uint32_t addr = prow + (((ch ^ row) & 7) << 4);
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(pk[h2 * 4 + 0]),
+                       "r"(pk[h2 * 4 + 1]), "r"(pk[h2 * 4 + 2]), "r"(pk[h2 * 4 + 3])
+                       : "memory");
+        }
+      }
+      l_sum = l_sum * alpha + rs;
+      sm100::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.s_free[sb]));
+      sm100::fence_proxy_async_smem();
+      // Raise O to the new maximum (rare): needs the previous PV product done.
+      if (j > 0 && __any_sync(adt::kFullMask, need)) {
+        if (!__all_sync(adt::kFullMask,
+                        wait_bar(&bars.pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, &s_abort, p.err)))
+          break;
+        sm100::tc_fence_after();
+#pragma unroll 1
+        for (int c0 = 0; c0 < D; c0 += 16) {
+          uint32_t o[16];
+          sm100::tmem_ld16(tmem + lane_base + kOCol + c0, o);
+          sm100::tmem_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 16; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+          sm100::tmem_st16(tmem + lane_base + kOCol + c0, o);
+        }
+        sm100::tmem_wait_st();
+      }
+      m_used = new_m;
+      sm100::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.p_full[sb]));
     }
   }
-  cp_async_wait<0>();
 
-  // Partial (m, l, O) of this split.
-  l0 += __shfl_xor_sync(adt::kFullMask, l0, 1);
-  l0 += __shfl_xor_sync(adt::kFullMask, l0, 2);
-  l1 += __shfl_xor_sync(adt::kFullMask, l1, 1);
-  l1 += __shfl_xor_sync(adt::kFullMask, l1, 2);
+  // ------------------------------------------------------------ epilogue
+  // Park this split's partial (O unnormalised, m, l) in shared memory (the
+  // stage ring is idle once O is complete), then merge.
+  constexpr int MS = C::kMergeStride;
+  float* so = reinterpret_cast<float*>(sStage);                         // [64][MS]
+  float2* sml = reinterpret_cast<float2*>(sStage + kMaxNodes * MS * 4);  // [64]
+  float* sw = reinterpret_cast<float*>(sStage + kMaxNodes * MS * 4 + kMaxNodes * 8);  // weights
+  if (warp < kSoftmaxWarps) {
+    // A split without key units (kv_len shorter than max_kv) contributes
+    // nothing: weight 0, zero partial.
+    const bool ok = nu > 0 && !s_abort && __all_sync(adt::kFullMask, wait_bar(&bars.o_full, 0, &s_abort, p.err));
+    if (!ok && lane < 16 && row < n) {
+      for (int c = 0; c < D; c += 4) *reinterpret_cast<float4*>(so + row * MS + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+      sml[row] = make_float2(-INFINITY, 0.f);
+    }
+    if (ok) {
+      sm100::tc_fence_after();
+      const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
+#pragma unroll
+      for (int c0 = 0; c0 < D; c0 += 16) {
+        uint32_t o[16];
+        sm100::tmem_ld16(tmem + lane_base + kOCol + c0, o);
+        sm100::tmem_wait_ld();
+        if (lane < 16 && row < n) {
+#pragma unroll
+          for (int e = 0; e < 16; e += 4)
+            *reinterpret_cast<float4*>(so + row * MS + c0 + e) =
+                make_float4(__uint_as_float(o[e]), __uint_as_float(o[e + 1]), __uint_as_float(o[e + 2]),
+                            __uint_as_float(o[e + 3]));
+        }
+      }
+      if (lane < 16 && row < n) sml[row] = make_float2(m_used, l_sum);
+    }
+  }
+  sm100::tc_fence_before();
+  __syncthreads();
+  if (warp == 0) sm100::tmem_dealloc(tmem, kTmemCols);
+
   const int64_t bh = static_cast<int64_t>(b) * p.H + h;
+  constexpr int kC4 = D / 4;
+  if (p.cluster_merge) {
+    // CTA r of the cluster merges rows r, r + S, ... from every peer's partial.
+    cg::cluster_group cl = cg::this_cluster();
+    cl.sync();
+    const int rank = static_cast<int>(cl.block_rank());
+    const int rows_mine = rank < n ? (n - rank + S - 1) / S : 0;
+    if (tid < rows_mine) {
+      const int rr = rank + S * tid;
+      float M = -INFINITY;
+      for (int c = 0; c < S; ++c) M = fmaxf(M, cl.map_shared_rank(sml, c)[rr].x);
+      float lt = 0.f;
+      for (int c = 0; c < S; ++c) {
+        const float2 ml = cl.map_shared_rank(sml, c)[rr];
+        const float w = ml.x == -INFINITY ? 0.f : exp2f(ml.x - M);
+        sw[tid * S + c] = w;
+        lt += w * ml.y;
+      }
+      const float inv = 1.f / lt;
+      for (int c = 0; c < S; ++c) sw[tid * S + c] *= inv;
+      if (p.lse) p.lse[static_cast<int64_t>(node0 + rr) * p.H + h] = (M + log2f(lt)) * kLn2;
+    }
+    __syncthreads();
+    for (int idx = tid; idx < rows_mine * kC4; idx += kThreads) {
+      const int i = idx / kC4, c4 = idx % kC4;
+      const int rr = rank + S * i;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int c = 0; c < S; ++c) {
+        const float w = sw[i * S + c];
+        if (w == 0.f) continue;
+        const float4 v = *reinterpret_cast<const float4*>(cl.map_shared_rank(so, c) + rr * MS + c4 * 4);
+        acc.x += w * v.x;
+        acc.y += w * v.y;
+        acc.z += w * v.z;
+        acc.w += w * v.w;
+      }
+      __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + rr) * p.H + h) * D + c4 * 4;
+      uint2 pk;
+      pk.x = pack_bf16x2(acc.x, acc.y);
+      pk.y = pack_bf16x2(acc.z, acc.w);
+      *reinterpret_cast<uint2*>(dst) = pk;
+    }
+    cl.sync();  // peers may still be reading this CTA's partial
+    return;
+  }
+
+  // More splits than a portable cluster holds: partials go to the workspace
+  // and the CTA that finishes a (tree, head) last merges them.
   float* po = p.part_o + (bh * S + split) * kMaxNodes * D;
   float2* pml = p.part_ml + (bh * S + split) * kMaxNodes;
-  if (warp_active) {
-#pragma unroll
-    for (int t = 0; t < C::kNTiles; ++t) {
-      const int d = t * 8 + tig * 2;
-      if (r0 < n) *reinterpret_cast<float2*>(po + r0 * D + d) = make_float2(o[t][0], o[t][1]);
-      if (r1 < n) *reinterpret_cast<float2*>(po + r1 * D + d) = make_float2(o[t][2], o[t][3]);
-    }
-    if (tig == 0) {
-      if (r0 < n) pml[r0] = make_float2(m0, l0);
-      if (r1 < n) pml[r1] = make_float2(m1, l1);
-    }
+  for (int idx = tid; idx < n * kC4; idx += kThreads) {
+    const int rr = idx / kC4, c4 = idx % kC4;
+    *reinterpret_cast<float4*>(po + rr * D + c4 * 4) = *reinterpret_cast<const float4*>(so + rr * MS + c4 * 4);
   }
+  if (tid < n) pml[tid] = sml[tid];
   __threadfence();
   __syncthreads();
-  if (tid == 0) {
-    const unsigned prev = atomicAdd(p.tickets + bh, 1u);
-    s_last = (prev == static_cast<unsigned>(S - 1));
-  }
+  if (tid == 0) s_last = atomicAdd(p.tickets + bh, 1u) == static_cast<unsigned>(S - 1);
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-
-  // Merge the splits of this (tree, head).
   const float* po_bh = p.part_o + bh * S * kMaxNodes * D;
   const float2* pml_bh = p.part_ml + bh * S * kMaxNodes;
-  constexpr int kC4 = D / 4;
-  for (int idx = tid; idx < n * kC4; idx += kThreads) {
-    const int row = idx / kC4, c4 = idx % kC4;
+  float* wsm = reinterpret_cast<float*>(sStage);  // [64][S]; the parked partial is in global now
+  __syncthreads();
+  if (tid < n) {
     float M = -INFINITY;
-    for (int sp = 0; sp < S; ++sp) M = fmaxf(M, __ldcg(&pml_bh[sp * kMaxNodes + row]).x);
+    for (int sp = 0; sp < S; ++sp) M = fmaxf(M, __ldcg(&pml_bh[sp * kMaxNodes + tid]).x);
     float lt = 0.f;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int sp = 0; sp < S; ++sp) {
-      const float2 ml = __ldcg(&pml_bh[sp * kMaxNodes + row]);
-      if (ml.x == -INFINITY) continue;
-      const float w = exp2f(ml.x - M);
+      const float2 ml = __ldcg(&pml_bh[sp * kMaxNodes + tid]);
+      const float w = ml.x == -INFINITY ? 0.f : exp2f(ml.x - M);
+      wsm[tid * S + sp] = w;
       lt += w * ml.y;
-      const float4 v = __ldcg(reinterpret_cast<const float4*>(po_bh + (sp * kMaxNodes + row) * D) + c4);
+    }
+    const float inv = 1.f / lt;
+    for (int sp = 0; sp < S; ++sp) wsm[tid * S + sp] *= inv;
+    if (p.lse) p.lse[static_cast<int64_t>(node0 + tid) * p.H + h] = (M + log2f(lt)) * kLn2;
+  }
+  __syncthreads();
+  constexpr int kStride4 = kMaxNodes * D / 4;
+  for (int idx = tid; idx < n * kC4; idx += kThreads) {
+    const int rr = idx / kC4, c4 = idx % kC4;
+    const float4* src = reinterpret_cast<const float4*>(po_bh + rr * D) + c4;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    int sp = 0;
+    for (; sp + 4 <= S; sp += 4) {
+      float4 v[4];
+#pragma unroll
+      for (int q4 = 0; q4 < 4; ++q4) v[q4] = __ldcg(src + (sp + q4) * kStride4);
+#pragma unroll
+      for (int q4 = 0; q4 < 4; ++q4) {
+        const float w = wsm[rr * S + sp + q4];
+        acc.x += w * v[q4].x;
+        acc.y += w * v[q4].y;
+        acc.z += w * v[q4].z;
+        acc.w += w * v[q4].w;
+      }
+    }
+    for (; sp < S; ++sp) {
+      const float4 v = __ldcg(src + sp * kStride4);
+      const float w = wsm[rr * S + sp];
       acc.x += w * v.x;
       acc.y += w * v.y;
       acc.z += w * v.z;
       acc.w += w * v.w;
     }
-    const float inv = 1.f / lt;
-    __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + row) * p.H + h) * D + c4 * 4;
-    __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
-    __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
+    __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + rr) * p.H + h) * D + c4 * 4;
     uint2 pk;
-    pk.x = *reinterpret_cast<uint32_t*>(&lo);
-    pk.y = *reinterpret_cast<uint32_t*>(&hi);
+    pk.x = pack_bf16x2(acc.x, acc.y);
+    pk.y = pack_bf16x2(acc.z, acc.w);
     *reinterpret_cast<uint2*>(dst) = pk;
-    if (c4 == 0 && p.lse) p.lse[static_cast<int64_t>(node0 + row) * p.H + h] = (M + log2f(lt)) * kLn2;
   }
   if (tid == 0) p.tickets[bh] = 0u;
 }
 
-int choose_splits(int sm_count, int B, int H, int D, int max_kv) {
-  const int units = (max_kv + kKeys - 1) / kKeys + 1;
-  const int per_sm = D == 128 ? 2 : 4;
-  const int target = sm_count * per_sm;
-  int s = target / (B * H);
+// ---------------------------------------------------------------- host side
+
+// Splits per (tree, head): about one CTA per SM, at most one split per unit
+// of keys.  Up to kMaxClusterSplits splits form a cluster; the count is
+// lowered until all B*H clusters are co-resident (GPC sizes decide how many
+// clusters of a given size fit at once).  Many splits (small B*H, long
+// prefixes) merge through the workspace instead.
+int max_active_clusters(int D, int cluster, int dev);
+
+int choose_splits(int sm_count, int B, int H, int D, int max_kv, int dev) {
+  const int units = (max_kv + kUnit - 1) / kUnit + 1;
+  const int bh = B * H;
+  int s = sm_count / bh;
   if (s < 1) s = 1;
   if (s > units) s = units;
+  if (s >= 2 * kMaxClusterSplits) return s > kMaxSplits ? kMaxSplits : s;
+  if (s > kMaxClusterSplits) s = kMaxClusterSplits;
+  while (s > 1 && max_active_clusters(D, s, dev) < bh) --s;
   return s;
 }
 
@@ -414,19 +638,149 @@ WsLayout ws_layout(int B, int H, int D, int splits) {
   return w;
 }
 
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+std::once_flag g_encode_once;
+EncodeTiledFn g_encode = nullptr;
+
+void load_encode() {
+  void* fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+          cudaSuccess &&
+      q == cudaDriverEntryPointSuccess)
+    g_encode = reinterpret_cast<EncodeTiledFn>(fn);
+}
+
+// 4-D map of a cache (d, pos, kv head, tree) with the 128-byte swizzle and
+// 64 x 64 boxes; positions at or past max_kv read as zero.
+adt_status make_cache_map(CUtensorMap* map, const void* base, int D, int max_kv, int Hkv, int B, int64_t sh,
+                          int64_t sb) {
+  std::call_once(g_encode_once, load_encode);
+  if (!g_encode) return ADT_ERR_CUDA;
+  const int64_t span = static_cast<int64_t>(max_kv > 0 ? max_kv : 1);
+  cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(span), static_cast<cuuint64_t>(Hkv),
+                        static_cast<cuuint64_t>(B)};
+  cuuint64_t strides[3] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(sh > 0 ? sh : span * D) * 2,
+                           static_cast<cuuint64_t>(sb > 0 ? sb : span * D * Hkv) * 2};
+  cuuint32_t box[4] = {64, kUnit, 1, 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? ADT_OK : ADT_ERR_INVALID_ARG;
+}
+
+int max_active_clusters(int D, int cluster, int dev) {
+  static int cache[64][2][kMaxClusterSplits + 1];  // 0 = not queried yet
+  int& slot = cache[dev & 63][D == 128 ? 1 : 0][cluster];
+  int v = __atomic_load_n(&slot, __ATOMIC_ACQUIRE);
+  if (v) return v - 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(cluster), 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(cluster);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int num = 0;
+  cudaError_t e;
+  if (D == 128) {
+    cudaFuncSetAttribute(tree_attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<128>::kDynSmem);
+    cfg.dynamicSmemBytes = Cfg<128>::kDynSmem;
+    e = cudaOccupancyMaxActiveClusters(&num, tree_attn_tc_kernel<128>, &cfg);
+  } else {
+    cudaFuncSetAttribute(tree_attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<64>::kDynSmem);
+    cfg.dynamicSmemBytes = Cfg<64>::kDynSmem;
+    e = cudaOccupancyMaxActiveClusters(&num, tree_attn_tc_kernel<64>, &cfg);
+  }
+  if (e != cudaSuccess) {
+    (void)cudaGetLastError();
+    num = 0;
+  }
+  __atomic_store_n(&slot, num + 1, __ATOMIC_RELEASE);
+  return num;
+}
+
 template <int D>
-adt_status launch(const AttnParams& prm, cudaStream_t st, int dev) {
+adt_status launch(TcParams prm, const void* k_cache, const void* v_cache, int64_t sb, int64_t sh, cudaStream_t st,
+                  int dev) {
   static unsigned configured[2] = {0u, 0u};  // bit per device (< 64)
   const unsigned bit = 1u << (dev & 31);
   unsigned& word = configured[dev >> 5];
   if (!(__atomic_load_n(&word, __ATOMIC_ACQUIRE) & bit)) {
-    ADT_CUDA_TRY(cudaFuncSetAttribute(tree_attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      Cfg<D>::kSmemBytes));
+    ADT_CUDA_TRY(cudaFuncSetAttribute(tree_attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      Cfg<D>::kDynSmem));
     __atomic_fetch_or(&word, bit, __ATOMIC_ACQ_REL);
   }
-  dim3 grid(prm.splits, prm.H, prm.B);
-  tree_attn_kernel<D><<<grid, kThreads, Cfg<D>::kSmemBytes, st>>>(prm);
+  CUtensorMap tm_k, tm_v;
+  adt_status s1 = make_cache_map(&tm_k, k_cache, D, prm.max_kv, prm.Hkv, prm.B, sh, sb);
+  if (s1 != ADT_OK) return s1;
+  s1 = make_cache_map(&tm_v, v_cache, D, prm.max_kv, prm.Hkv, prm.B, sh, sb);
+  if (s1 != ADT_OK) return s1;
+  prm.cluster_merge = prm.splits <= kMaxClusterSplits ? 1 : 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(prm.splits), static_cast<unsigned>(prm.H), static_cast<unsigned>(prm.B));
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = Cfg<D>::kDynSmem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = prm.cluster_merge ? static_cast<unsigned>(prm.splits) : 1u;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, tree_attn_tc_kernel<D>, tm_k, tm_v, prm));
   return adt::launch_status();
+}
+
+// Shared host checks of both entry points.
+adt_status check_args(const adt_bf16* q, const adt_bf16* k_cache, const adt_bf16* v_cache, const int32_t* kv_len,
+                      int64_t sb, int64_t sh, const adt_bf16* k_tree, const adt_bf16* v_tree,
+                      const int32_t* parents, const int32_t* node_offsets, int32_t B, int32_t H, int32_t Hkv,
+                      int32_t D, int32_t max_nodes, int32_t max_kv, float scale, const adt_bf16* out) {
+  ADT_REQUIRE(q && k_cache && v_cache && kv_len && k_tree && v_tree && parents && node_offsets && out);
+  ADT_REQUIRE(B >= 1 && H >= 1 && Hkv >= 1 && H % Hkv == 0);
+  ADT_REQUIRE(static_cast<int64_t>(B) * H <= kMaxBH && B <= 65535 && H <= 65535);
+  ADT_REQUIRE(max_nodes >= 1 && max_kv >= 0 && max_kv < (1 << 30));
+  ADT_REQUIRE(scale > 0.f && scale < 1e30f);
+  if (D != 64 && D != 128) return ADT_ERR_UNSUPPORTED;
+  if (max_nodes > kMaxNodes) return ADT_ERR_UNSUPPORTED;
+  ADT_REQUIRE(sb >= 0 && sh >= 0 && sb % 8 == 0 && sh % 8 == 0);
+  ADT_REQUIRE(Hkv == 1 || sh >= static_cast<int64_t>(max_kv) * D);
+  ADT_REQUIRE(B == 1 || sb >= static_cast<int64_t>(max_kv) * D);
+  ADT_REQUIRE(adt::aligned16(q) && adt::aligned16(k_cache) && adt::aligned16(v_cache) && adt::aligned16(k_tree) &&
+              adt::aligned16(v_tree) && adt::aligned16(out));
+  return ADT_OK;
+}
+
+TcParams make_params(const adt_bf16* q, const int32_t* kv_len, const adt_bf16* k_tree, const adt_bf16* v_tree,
+                     const int32_t* parents, const int32_t* node_offsets, int B, int H, int Hkv, int max_kv,
+                     int splits, float scale, adt_bf16* out, float* lse, unsigned* err) {
+  TcParams prm{};
+  prm.q = reinterpret_cast<const __nv_bfloat16*>(q);
+  prm.kt = reinterpret_cast<const __nv_bfloat16*>(k_tree);
+  prm.vt = reinterpret_cast<const __nv_bfloat16*>(v_tree);
+  prm.kv_len = kv_len;
+  prm.parents = parents;
+  prm.offs = node_offsets;
+  prm.B = B;
+  prm.H = H;
+  prm.Hkv = Hkv;
+  prm.group = H / Hkv;
+  prm.max_kv = max_kv;
+  prm.splits = splits;
+  prm.scale_log2 = scale * kLog2e;
+  prm.out = reinterpret_cast<__nv_bfloat16*>(out);
+  prm.lse = lse;
+  prm.err = err;
+  return prm;
 }
 
 }  // namespace
@@ -439,7 +793,7 @@ size_t adt_tree_attn_workspace_size(int32_t B, int32_t H, int32_t D, int32_t max
   if (B < 1 || H < 1 || (D != 64 && D != 128) || max_kv < 0 || static_cast<int64_t>(B) * H > kMaxBH) return 0;
   adt::DeviceInfo info;
   if (adt::device_info(&info) != ADT_OK) return 0;
-  return ws_layout(B, H, D, choose_splits(info.sm_count, B, H, D, max_kv)).total;
+  return ws_layout(B, H, D, choose_splits(info.sm_count, B, H, D, max_kv, info.device)).total;
 }
 
 adt_status adt_tree_attn(const adt_bf16* q, const adt_bf16* k_cache, const adt_bf16* v_cache,
@@ -448,50 +802,24 @@ adt_status adt_tree_attn(const adt_bf16* q, const adt_bf16* k_cache, const adt_b
                          const int32_t* node_offsets, int32_t B, int32_t H, int32_t Hkv, int32_t D,
                          int32_t max_nodes, int32_t max_kv, float softmax_scale, adt_bf16* out,
                          float* lse, void* workspace, size_t workspace_bytes, void* stream) {
-  ADT_REQUIRE(q && k_cache && v_cache && kv_len && k_tree && v_tree && parents && node_offsets && out);
-  ADT_REQUIRE(B >= 1 && H >= 1 && Hkv >= 1 && H % Hkv == 0);
-  ADT_REQUIRE(static_cast<int64_t>(B) * H <= kMaxBH && B <= 65535 && H <= 65535);
-  ADT_REQUIRE(max_nodes >= 1 && max_kv >= 0);
-  ADT_REQUIRE(softmax_scale > 0.f && softmax_scale < 1e30f);
-  if (D != 64 && D != 128) return ADT_ERR_UNSUPPORTED;
-  if (max_nodes > kMaxNodes) return ADT_ERR_UNSUPPORTED;
-  ADT_REQUIRE(cache_stride_b >= 0 && cache_stride_h >= 0 && cache_stride_b % 8 == 0 &&
-              cache_stride_h % 8 == 0);
-  ADT_REQUIRE(adt::aligned16(q) && adt::aligned16(k_cache) && adt::aligned16(v_cache) &&
-              adt::aligned16(k_tree) && adt::aligned16(v_tree) && adt::aligned16(out));
-  adt::DeviceInfo info;
-  adt_status st = adt::device_info(&info);
+  adt_status st = check_args(q, k_cache, v_cache, kv_len, cache_stride_b, cache_stride_h, k_tree, v_tree, parents,
+                             node_offsets, B, H, Hkv, D, max_nodes, max_kv, softmax_scale, out);
   if (st != ADT_OK) return st;
-  const int splits = choose_splits(info.sm_count, B, H, D, max_kv);
+  adt::DeviceInfo info;
+  st = adt::device_info(&info);
+  if (st != ADT_OK) return st;
+  const int splits = choose_splits(info.sm_count, B, H, D, max_kv, info.device);
   const WsLayout w = ws_layout(B, H, D, splits);
   if (!workspace || workspace_bytes < w.total || !adt::aligned16(workspace)) return ADT_ERR_WORKSPACE;
   uint8_t* ws = static_cast<uint8_t*>(workspace);
-  AttnParams prm;
-  prm.q = reinterpret_cast<const __nv_bfloat16*>(q);
-  prm.kc = reinterpret_cast<const __nv_bfloat16*>(k_cache);
-  prm.vc = reinterpret_cast<const __nv_bfloat16*>(v_cache);
-  prm.kv_len = kv_len;
-  prm.sb = cache_stride_b;
-  prm.sh = cache_stride_h;
-  prm.kt = reinterpret_cast<const __nv_bfloat16*>(k_tree);
-  prm.vt = reinterpret_cast<const __nv_bfloat16*>(v_tree);
-  prm.parents = parents;
-  prm.offs = node_offsets;
-  prm.B = B;
-  prm.H = H;
-  prm.Hkv = Hkv;
-  prm.group = H / Hkv;
-  prm.max_kv = max_kv;
-  prm.splits = splits;
-  prm.scale_log2 = softmax_scale * kLog2e;
-  prm.out = reinterpret_cast<__nv_bfloat16*>(out);
-  prm.lse = lse;
+  TcParams prm = make_params(q, kv_len, k_tree, v_tree, parents, node_offsets, B, H, Hkv, max_kv, splits,
+                             softmax_scale, out, lse, info.error_word);
   prm.part_o = reinterpret_cast<float*>(ws + w.part_o);
   prm.part_ml = reinterpret_cast<float2*>(ws + w.part_ml);
   prm.tickets = reinterpret_cast<unsigned*>(ws + w.tickets);
-  prm.err = info.error_word;
   cudaStream_t s = adt::as_stream(stream);
-  return D == 128 ? launch<128>(prm, s, info.device) : launch<64>(prm, s, info.device);
+  return D == 128 ? launch<128>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device)
+                  : launch<64>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device);
 }
 
 }  // extern "C"
@@ -501,11 +829,10 @@ adt_status adt_tree_attn(const adt_bf16* q, const adt_bf16* k_cache, const adt_b
 // allocate device memory themselves, for example a plugin inside a serving
 // engine whose host owns every device allocation, or code on a latency-
 // critical thread that must not call cudaMalloc (it can synchronise the
-// device).  The split partials and completion tickets live in one fixed,
-// per-device static array instead of a caller-provided workspace.
+// device).  The scratch that adt_tree_attn takes as a workspace (split
+// partials and completion tickets) lives in one fixed, per-device static
+// array instead.
 // ---------------------------------------------------------------------------
-
-#include <mutex>
 
 // 8 MiB of scratch, held by every GPU that loads the library until the
 // process exits.  Shared by all calls on a device: calls that overlap on the
@@ -553,26 +880,18 @@ extern "C" adt_status adt_tree_attn_noalloc(const adt_bf16* q, const adt_bf16* k
                                             int32_t B, int32_t H, int32_t Hkv, int32_t D,
                                             int32_t max_nodes, int32_t max_kv, float softmax_scale,
                                             adt_bf16* out, float* lse, void* stream) {
-  ADT_REQUIRE(q && k_cache && v_cache && kv_len && k_tree && v_tree && parents && node_offsets && out);
-  ADT_REQUIRE(B >= 1 && H >= 1 && Hkv >= 1 && H % Hkv == 0);
-  ADT_REQUIRE(B <= 65535 && H <= 65535);
-  ADT_REQUIRE(max_nodes >= 1 && max_kv >= 0);
-  ADT_REQUIRE(softmax_scale > 0.f && softmax_scale < 1e30f);
-  if (D != 64 && D != 128) return ADT_ERR_UNSUPPORTED;
-  if (max_nodes > kMaxNodes) return ADT_ERR_UNSUPPORTED;
-  ADT_REQUIRE(cache_stride_b >= 0 && cache_stride_h >= 0 && cache_stride_b % 8 == 0 &&
-              cache_stride_h % 8 == 0);
-  ADT_REQUIRE(adt::aligned16(q) && adt::aligned16(k_cache) && adt::aligned16(v_cache) &&
-              adt::aligned16(k_tree) && adt::aligned16(v_tree) && adt::aligned16(out));
+  adt_status st = check_args(q, k_cache, v_cache, kv_len, cache_stride_b, cache_stride_h, k_tree, v_tree, parents,
+                             node_offsets, B, H, Hkv, D, max_nodes, max_kv, softmax_scale, out);
+  if (st != ADT_OK) return st;
   adt::DeviceInfo info;
-  adt_status st = adt::device_info(&info);
+  st = adt::device_info(&info);
   if (st != ADT_OK) return st;
   if (info.device < 0 || info.device >= kNoAllocMaxDevices) return ADT_ERR_UNSUPPORTED;
   std::call_once(g_noalloc_once[info.device], noalloc_setup, info.device);
   if (g_noalloc_status[info.device] != cudaSuccess || !g_noalloc_ptr[info.device]) return ADT_ERR_CUDA;
   // As many splits as the usual heuristic picks, fewer if the partials would
   // not fit; a shape that does not fit even unsplit is rejected.
-  int splits = choose_splits(info.sm_count, B, H, D, max_kv);
+  int splits = choose_splits(info.sm_count, B, H, D, max_kv, info.device);
   while (splits > 1 && noalloc_layout(B, H, D, splits).total > kNoAllocScratchBytes) --splits;
   const NoAllocLayout w = noalloc_layout(B, H, D, splits);
   if (w.total > kNoAllocScratchBytes) return ADT_ERR_WORKSPACE;
@@ -580,29 +899,11 @@ extern "C" adt_status adt_tree_attn_noalloc(const adt_bf16* q, const adt_bf16* k
   cudaStream_t s = adt::as_stream(stream);
   // The array keeps the previous call's contents: the tickets must start at zero.
   ADT_CUDA_TRY(cudaMemsetAsync(ws + w.tickets, 0, static_cast<size_t>(B) * H * sizeof(unsigned), s));
-  AttnParams prm;
-  prm.q = reinterpret_cast<const __nv_bfloat16*>(q);
-  prm.kc = reinterpret_cast<const __nv_bfloat16*>(k_cache);
-  prm.vc = reinterpret_cast<const __nv_bfloat16*>(v_cache);
-  prm.kv_len = kv_len;
-  prm.sb = cache_stride_b;
-  prm.sh = cache_stride_h;
-  prm.kt = reinterpret_cast<const __nv_bfloat16*>(k_tree);
-  prm.vt = reinterpret_cast<const __nv_bfloat16*>(v_tree);
-  prm.parents = parents;
-  prm.offs = node_offsets;
-  prm.B = B;
-  prm.H = H;
-  prm.Hkv = Hkv;
-  prm.group = H / Hkv;
-  prm.max_kv = max_kv;
-  prm.splits = splits;
-  prm.scale_log2 = softmax_scale * kLog2e;
-  prm.out = reinterpret_cast<__nv_bfloat16*>(out);
-  prm.lse = lse;
+  TcParams prm = make_params(q, kv_len, k_tree, v_tree, parents, node_offsets, B, H, Hkv, max_kv, splits,
+                             softmax_scale, out, lse, info.error_word);
   prm.part_o = reinterpret_cast<float*>(ws + w.part_o);
   prm.part_ml = reinterpret_cast<float2*>(ws + w.part_ml);
   prm.tickets = reinterpret_cast<unsigned*>(ws + w.tickets);
-  prm.err = info.error_word;
-  return D == 128 ? launch<128>(prm, s, info.device) : launch<64>(prm, s, info.device);
+  return D == 128 ? launch<128>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device)
+                  : launch<64>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device);
 }

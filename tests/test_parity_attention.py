@@ -55,7 +55,7 @@ def test_batch_of_eight_ragged_prefixes():
     g = np.random.default_rng(5)
     kv = g.integers(600, 2401, size=8).tolist()
     sizes = g.integers(8, 65, size=8).tolist()
-    case = AttnCase(sizes, kv, 8, 8, 128, seed=77, max_depth=10, max_children=8)
+    case = AttnCase(sizes, kv, 8, 8, 128, seed=77, max_depth=10, max_children=8, lmax=2400 + 8)
     got, _, _ = case.run_gpu(max_nodes=64, max_kv=2400)
     ref, _ = case.run_oracle()
     assert_attention_close(got, ref)

@@ -64,5 +64,6 @@ def test_noalloc_rejects_a_shape_beyond_its_scratch():
     t = torch.zeros(64, dtype=torch.int32, device="cuda")
     p = _ptr(t)
     stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
-    st = B.lib().adt_tree_attn_noalloc(p, p, p, p, 0, 0, p, p, p, p, 64, 64, 64, 128, 64, 100, 0.1, p, None, stream)
+    sh, sb = 100 * 128, 64 * 100 * 128  # strides of a [64][64][100][128] cache
+    st = B.lib().adt_tree_attn_noalloc(p, p, p, p, sb, sh, p, p, p, p, 64, 64, 64, 128, 64, 100, 0.1, p, None, stream)
     assert st == 5  # ADT_ERR_WORKSPACE, nothing launched
