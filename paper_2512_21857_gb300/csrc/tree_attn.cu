@@ -16,12 +16,13 @@
 //   warp 5    one elected thread issues tcgen05.mma: S = Q K^T into a
 //             double-buffered tensor-memory tile (M = 64 queries, N = 64
 //             keys), then O += P V (N = head_dim, V read MN-major);
-//   warps 0-3 softmax: each thread owns one query row (tensor-memory lane
-//             32w + i holds row 16w + i for M = 64), reads its S row,
-//             masks, exponentiates with a lazily raised running maximum
-//             (O is rescaled only when the maximum grows by more than 2^8),
-//             writes P (bf16) to shared memory for the PV product; at the
-//             end they read O and l and emit the split's partial.
+//   warps 0-3 softmax: warp w owns query rows 16w .. 16w+15 (tensor-memory
+//             lanes 32w .. 32w+15 for M = 64), read with the 16x256b shape so
+//             that each thread holds two rows x 16 columns of a chunk; masks
+//             branch-free, exponentiates against a lazily raised running
+//             maximum (O is rescaled only when a row maximum grows by more
+//             than 2^8), writes P (bf16) to shared memory for the PV
+//             product; at the end they read O and l and emit the partial.
 // mbarriers connect the roles; every wait is bounded and a timeout sets
 // ADT_DEVERR_TIMEOUT.  The splits of one (tree, head) form a thread-block
 // cluster (<= 8) and merge their partials through distributed shared
@@ -59,11 +60,11 @@ struct Cfg {
   static constexpr int kBlocks = D / 64;             // 128-byte column blocks per row
   static constexpr int kBlockBytes = kUnit * 128;    // one column block of 64 rows
   static constexpr int kTileBytes = kBlocks * kBlockBytes;  // 64 rows x D bf16
-  static constexpr int kStages = D == 128 ? 5 : 8;
+  static constexpr int kStages = D == 128 ? 4 : 8;
   static constexpr int kQOff = 0;
   static constexpr int kPOff = kTileBytes;                  // two P buffers (64 x 64 bf16)
-  static constexpr int kTrashOff = kPOff + 2 * kBlockBytes; // 16 scratch rows for idle lanes
-  static constexpr int kStageOff = kTrashOff + 2048;
+  static constexpr int kTreeOff = kPOff + 2 * kBlockBytes;    // tree unit: K tile, then V tile
+  static constexpr int kStageOff = kTreeOff + 2 * kTileBytes;
   static constexpr int kStageBytes = 2 * kTileBytes;        // K tile, then V tile
   static constexpr int kDynSmem = kStageOff + kStages * kStageBytes + 1024;  // + alignment slack
   static constexpr uint32_t kIdescS = sm100::idesc_bf16_f32(64, 64, 0, 0);
@@ -103,6 +104,40 @@ __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wai
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
+}
+
+
+// tcgen05.ld / st, shape 16x256b, 8 repetitions: for an M = 64 accumulator
+// (rows 16w .. 16w+15 in lanes 32w .. 32w+15), thread (g = lane / 4,
+// t = lane % 4) of warp w gets, for each 8-column block b = 0..7 starting at
+// the address's column: r[4b + 0, 1] = row 16w + g, columns 8b + 2t, 8b + 2t + 1
+// and r[4b + 2, 3] = the same columns of row 16w + g + 8.
+__device__ __forceinline__ void tmem_ld_16x256b_x8(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.16x256b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
+}
+__device__ __forceinline__ void tmem_st_16x256b_x8(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.16x256b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};\n" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+      "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]),
+      "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]),
+      "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+
+// x masked to -inf where the keep bit is 0, without branching.
+__device__ __forceinline__ float mask_or_neg_inf(float x, uint32_t keep_bit) {
+  const uint32_t keep = 0u - keep_bit;
+  return __uint_as_float((__float_as_uint(x) & keep) | (0xFF800000u & ~keep));
 }
 
 struct Barriers {
@@ -200,12 +235,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int u_begin = static_cast<int>(static_cast<int64_t>(split) * U / S);
   const int u_end = static_cast<int>(static_cast<int64_t>(split + 1) * U / S);
   const int nu = u_end - u_begin;
+  // The CTA whose share ends with the tree unit processes it first (its K/V
+  // are loaded with Q at the start); prefix units follow in order through
+  // the TMA ring.  Iteration j handles unit unit_of(j).
+  const int has_tree = (u_end == U && nu > 0) ? 1 : 0;
+  const int np = nu - has_tree;  // prefix units of this CTA
+  auto unit_of = [&](int j) { return has_tree ? (j == 0 ? U - 1 : u_begin + j - 1) : u_begin + j; };
   const int NS = C::kStages;
 
   uint8_t* sQ = smem + C::kQOff;
   uint8_t* sP = smem + C::kPOff;
   uint8_t* sStage = smem + C::kStageOff;
-  uint8_t* sTrash = smem + C::kTrashOff;
+  uint8_t* sTree = smem + C::kTreeOff;
 
   if (tid == 0) {
     sm100::mbar_init(sm100::smem_addr(&bars.q_full), kSoftmaxWarps);
@@ -231,39 +272,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   sm100::tc_fence_after();
   const uint32_t tmem = tmem_slot;
 
-  // Per-row state of the softmax threads (lane < 16 of warps 0-3).
-  const int row = warp * 16 + lane;
-  float m_used = -INFINITY, l_sum = 0.f;
+  // Final row statistics of the softmax threads' two rows (a, b).
+  float m_ra = -INFINITY, l_ra = 0.f, m_rb = -INFINITY, l_rb = 0.f;
 
   if (warp == kProducerWarp) {
     // ------------------------------------------------------------ producer
     int issued = 0;
-    for (int j = 0; j < nu; ++j) {
-      const int st = j % NS;
-      if (j >= NS &&
-          !__all_sync(adt::kFullMask, wait_bar(&bars.kv_empty[st], ((j / NS) - 1) & 1, &s_abort, p.err)))
+    for (int jp = 0; jp < np; ++jp) {
+      const int st = jp % NS;
+      if (jp >= NS &&
+          !__all_sync(adt::kFullMask, wait_bar(&bars.kv_empty[st], ((jp / NS) - 1) & 1, &s_abort, p.err)))
         break;
-      uint8_t* kdst = sStage + st * C::kStageBytes;
-      uint8_t* vdst = kdst + C::kTileBytes;
-      const int u = u_begin + j;
-      if (u == U - 1) {
-        // Tree unit: rows node0 .. node0+63 of k_tree / v_tree for kv head g;
-        // rows past this tree are zero-filled, never read out of bounds.
-        for (int i = lane; i < kUnit * (D / 8); i += 32) {
-          const int r = i / (D / 8), ch = i % (D / 8);
-          const bool valid = r < n;
-          const int64_t off = (static_cast<int64_t>(node0 + (valid ? r : 0)) * p.Hkv + g) * D + ch * 8;
-          cp_async16(sm100::smem_addr(kdst) + sw128_off(r, ch), p.kt + off, valid ? 16 : 0);
-          cp_async16(sm100::smem_addr(vdst) + sw128_off(r, ch), p.vt + off, valid ? 16 : 0);
-        }
-        cp_async_wait_all();
-        sm100::fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.kv_full[st]));
-      } else if (lane == 0) {
+      if (lane == 0) {
+        uint8_t* kdst = sStage + st * C::kStageBytes;
+        uint8_t* vdst = kdst + C::kTileBytes;
         const uint32_t bar = sm100::smem_addr(&bars.kv_full[st]);
         sm100::mbar_arrive_expect_tx(bar, 2 * C::kTileBytes);
-        const int key0 = u * kUnit;
+        const int key0 = (u_begin + jp) * kUnit;
         for (int blk = 0; blk < C::kBlocks; ++blk) {
           sm100::tma_load_4d(sm100::smem_addr(kdst + blk * C::kBlockBytes), &tm_k, blk * 64, key0, g, b, bar);
           sm100::tma_load_4d(sm100::smem_addr(vdst + blk * C::kBlockBytes), &tm_v, blk * 64, key0, g, b, bar);
@@ -274,8 +299,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (s_abort && lane == 0) {
       // let every copy still in flight land before the CTA can exit
-      for (int j = (issued > NS ? issued - NS : 0); j < issued; ++j)
-        (void)sm100::mbar_wait_bounded(sm100::smem_addr(&bars.kv_full[j % NS]), (j / NS) & 1, kWaitLimit);
+      for (int jp = (issued > NS ? issued - NS : 0); jp < issued; ++jp)
+        (void)sm100::mbar_wait_bounded(sm100::smem_addr(&bars.kv_full[jp % NS]), (jp / NS) & 1, kWaitLimit);
     }
   } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
@@ -287,23 +312,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int pb = i & 1;
         if (!wait_bar(&bars.p_full[pb], (i >> 1) & 1, &s_abort, p.err)) return false;
         sm100::tc_fence_after();
-        const uint32_t v_addr = sm100::smem_addr(sStage + (i % NS) * C::kStageBytes + C::kTileBytes);
+        const bool tree_i = has_tree && i == 0;
+        const int ip = i - has_tree;
+        const uint32_t v_addr = tree_i ? sm100::smem_addr(sTree + C::kTileBytes)
+                                       : sm100::smem_addr(sStage + (ip % NS) * C::kStageBytes + C::kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < kUnit / 16; ++kk) {
           const uint64_t da = sm100::smem_desc_sw128(p_addr + pb * C::kBlockBytes + kk * 32, 16, 1024);
           const uint64_t db = sm100::smem_desc_sw128(v_addr + kk * 2048, C::kBlockBytes, 1024);
           sm100::mma_bf16_ss(tmem + kOCol, da, db, C::kIdescO, (i > 0 || kk > 0) ? 1u : 0u);
         }
-        sm100::mma_commit(sm100::smem_addr(&bars.kv_empty[i % NS]));
+        if (!tree_i) sm100::mma_commit(sm100::smem_addr(&bars.kv_empty[ip % NS]));
         sm100::mma_commit(sm100::smem_addr(&bars.pv_done[pb]));
         return true;
       };
       for (int j = 0; ok && j < nu; ++j) {
-        const int st = j % NS, sb = j & 1;
-        if (!wait_bar(&bars.kv_full[st], (j / NS) & 1, &s_abort, p.err)) break;
+        const bool tree_j = has_tree && j == 0;
+        const int jp = j - has_tree;
+        const int st = jp % NS, sb = j & 1;
+        if (!tree_j && !wait_bar(&bars.kv_full[st], (jp / NS) & 1, &s_abort, p.err)) break;
         if (j >= 2 && !wait_bar(&bars.s_free[sb], ((j >> 1) - 1) & 1, &s_abort, p.err)) break;
         sm100::tc_fence_after();
-        const uint32_t k_addr = sm100::smem_addr(sStage + st * C::kStageBytes);
+        const uint32_t k_addr = tree_j ? sm100::smem_addr(sTree) : sm100::smem_addr(sStage + st * C::kStageBytes);
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t off = (kk >> 2) * C::kBlockBytes + (kk & 3) * 32;
@@ -331,116 +361,147 @@ __global__ void __launch_bounds__(kThreads, 1)
       const __nv_bfloat16* src = p.q + (static_cast<int64_t>(node0 + (valid ? r : 0)) * p.H + h) * D + ch * 8;
       cp_async16(sm100::smem_addr(sQ) + sw128_off(r, ch), src, valid ? 16 : 0);
     }
+    if (has_tree) {
+      // Tree unit: rows node0 .. node0+63 of k_tree / v_tree for kv head g;
+      // rows past this tree are zero-filled, never read out of bounds.
+      for (int i = tid; i < kUnit * (D / 8); i += kSoftmaxWarps * 32) {
+        const int r = i / (D / 8), ch = i % (D / 8);
+        const bool valid = r < n;
+        const int64_t off = (static_cast<int64_t>(node0 + (valid ? r : 0)) * p.Hkv + g) * D + ch * 8;
+        cp_async16(sm100::smem_addr(sTree) + sw128_off(r, ch), p.kt + off, valid ? 16 : 0);
+        cp_async16(sm100::smem_addr(sTree + C::kTileBytes) + sw128_off(r, ch), p.vt + off, valid ? 16 : 0);
+      }
+    }
     cp_async_wait_all();
     sm100::fence_proxy_async_smem();
     __syncwarp();
     if (lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.q_full));
 
-    const bool rvalid = lane < 16 && row < n;
-    const uint64_t am = rvalid ? anc[row] : 0ull;
+    // Thread (g, t) = (lane / 4, lane % 4) of warp w owns rows ra = 16w + g
+    // and rb = ra + 8 of the tile, columns 8b + 2t, 8b + 2t + 1 of every
+    // 8-column block b (the 16x256b tensor-memory layout); the four threads
+    // of a quad share a row and combine row statistics with two shuffles.
+    const int g8 = lane >> 2, t4 = lane & 3;
+    const int ra = warp * 16 + g8, rb = ra + 8;
+    const uint64_t ama = ra < n ? anc[ra] : 0ull;
+    const uint64_t amb = rb < n ? anc[rb] : 0ull;
     const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
+    float mua = -INFINITY, mub = -INFINITY;  // running maxima used for the exponentials
+    float la = 0.f, lb = 0.f;                // this thread's share of the row sums
     for (int j = 0; j < nu; ++j) {
       const int sb = j & 1;
       if (!__all_sync(adt::kFullMask, wait_bar(&bars.s_full[sb], (j >> 1) & 1, &s_abort, p.err))) break;
       sm100::tc_fence_after();
-      const int u = u_begin + j;
-      // Which of the chunk's 64 keys this row sees: the prefix up to L, or
-      // the row's ancestors (and itself) in the tree unit.  Applied with
-      // integer bit operations so that no lane ever branches on it: the
-      // lanes of a warp hold different rows, and per-key branches would
-      // diverge.
-      uint64_t vm;
+      uint32_t r[32];
+      tmem_ld_16x256b_x8(tmem + lane_base + sb * 64, r);
+      sm100::tmem_wait_ld();
+      // S is in registers: hand the tensor-memory buffer back to the MMA warp.
+      sm100::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.s_free[sb]));
+
+      const int u = unit_of(j);
+      // Which of the chunk's 64 keys a row sees (the prefix up to L, or the
+      // row's ancestors and itself in the tree unit), applied with bit
+      // operations so no lane branches on it.
+      uint64_t vma, vmb;
       if (u == U - 1) {
-        vm = am;
+        vma = ama;
+        vmb = amb;
       } else {
         const int kl = L - u * kUnit;  // >= 1 for every prefix unit
-        vm = kl >= 64 ? ~0ull : ((1ull << kl) - 1ull);
+        vma = vmb = kl >= 64 ? ~0ull : ((1ull << kl) - 1ull);
       }
       const float scale = p.scale_log2;
-      const uint32_t s_addr = tmem + lane_base + sb * 64;
-      // Pass 1: row maximum of the masked, scaled scores, 16 columns at a
-      // time (the outer loops stay rolled so the hot code stays small).
-      float mx = -INFINITY;
-#pragma unroll 1
-      for (int g4 = 0; g4 < 4; ++g4) {
-        uint32_t r[16];
-        sm100::tmem_ld16(s_addr + g4 * 16, r);
-        sm100::tmem_wait_ld();
-        const uint32_t bits = static_cast<uint32_t>(vm >> (g4 * 16));
+      float xa[16], xb[16];
+      float mxa = -INFINITY, mxb = -INFINITY;
 #pragma unroll
-        for (int e = 0; e < 16; ++e) {
-          const uint32_t keep = 0u - ((bits >> e) & 1u);
-          const uint32_t xb = __float_as_uint(__uint_as_float(r[e]) * scale);
-          mx = fmaxf(mx, __uint_as_float((xb & keep) | (0xFF800000u & ~keep)));
+      for (int bk = 0; bk < 8; ++bk) {
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int c = 8 * bk + 2 * t4 + e;
+          xa[2 * bk + e] = mask_or_neg_inf(__uint_as_float(r[4 * bk + e]) * scale,
+                                           static_cast<uint32_t>(vma >> c) & 1u);
+          xb[2 * bk + e] = mask_or_neg_inf(__uint_as_float(r[4 * bk + 2 + e]) * scale,
+                                           static_cast<uint32_t>(vmb >> c) & 1u);
+          mxa = fmaxf(mxa, xa[2 * bk + e]);
+          mxb = fmaxf(mxb, xb[2 * bk + e]);
         }
       }
-      const bool need = lane < 16 && mx > m_used + kRescaleThreshold;
-      const float new_m = need ? mx : m_used;
-      const float alpha = need ? exp2f(m_used - new_m) : 1.f;
-      const float base = new_m == -INFINITY ? 0.f : new_m;
+      mxa = fmaxf(mxa, __shfl_xor_sync(adt::kFullMask, mxa, 1));
+      mxa = fmaxf(mxa, __shfl_xor_sync(adt::kFullMask, mxa, 2));
+      mxb = fmaxf(mxb, __shfl_xor_sync(adt::kFullMask, mxb, 1));
+      mxb = fmaxf(mxb, __shfl_xor_sync(adt::kFullMask, mxb, 2));
+      // Lazily raised maximum: O is rescaled only when a row's maximum grows
+      // by more than 2^8 over the one its exponentials were taken against.
+      const bool needa = mxa > mua + kRescaleThreshold, needb = mxb > mub + kRescaleThreshold;
+      const float nma = needa ? mxa : mua, nmb = needb ? mxb : mub;
+      const float alpha_a = needa ? exp2f(mua - nma) : 1.f, alpha_b = needb ? exp2f(mub - nmb) : 1.f;
+      const float base_a = nma == -INFINITY ? 0.f : nma, base_b = nmb == -INFINITY ? 0.f : nmb;
+      float rsa = 0.f, rsb = 0.f;
+      uint32_t pa[8], pb[8];
+#pragma unroll
+      for (int bk = 0; bk < 8; ++bk) {
+        const float a0 = exp2f(xa[2 * bk] - base_a), a1 = exp2f(xa[2 * bk + 1] - base_a);
+        const float b0 = exp2f(xb[2 * bk] - base_b), b1 = exp2f(xb[2 * bk + 1] - base_b);
+        rsa += a0 + a1;
+        rsb += b0 + b1;
+        pa[bk] = pack_bf16x2(a0, a1);
+        pb[bk] = pack_bf16x2(b0, b1);
+      }
+      la = la * alpha_a + rsa;
+      lb = lb * alpha_b + rsb;
       // P buffer sb was last read by the PV product of chunk j - 2.
       if (j >= 2 &&
           !__all_sync(adt::kFullMask, wait_bar(&bars.pv_done[sb], ((j >> 1) - 1) & 1, &s_abort, p.err)))
         break;
-      // Pass 2: p = 2^(s - base) (0 for masked keys), row sum, bf16 P row
-      // into shared memory; lanes 16-31 (no row of the M = 64 tile) write a
-      // scratch row instead of branching around the stores.
-      float rs = 0.f;
-      const uint32_t prow = lane < 16 ? sm100::smem_addr(sP + sb * C::kBlockBytes) + row * 128
-                                      : sm100::smem_addr(sTrash) + (lane - 16) * 128;
-#pragma unroll 1
-      for (int g4 = 0; g4 < 4; ++g4) {
-        uint32_t r[16];
-        sm100::tmem_ld16(s_addr + g4 * 16, r);
-        sm100::tmem_wait_ld();
-        const uint32_t bits = static_cast<uint32_t>(vm >> (g4 * 16));
-        uint32_t pk[8];
+      {
+        const uint32_t pbase = sm100::smem_addr(sP + sb * C::kBlockBytes);
+        const uint32_t rowa = pbase + ra * 128 + t4 * 4, rowb = pbase + rb * 128 + t4 * 4;
 #pragma unroll
-        for (int e = 0; e < 16; e += 2) {
-          const uint32_t k0 = 0u - ((bits >> e) & 1u), k1 = 0u - ((bits >> (e + 1)) & 1u);
-          const uint32_t x0 = __float_as_uint(__uint_as_float(r[e]) * scale);
-          const uint32_t x1 = __float_as_uint(__uint_as_float(r[e + 1]) * scale);
-          const float p0 = exp2f(__uint_as_float((x0 & k0) | (0xFF800000u & ~k0)) - base);
-          const float p1 = exp2f(__uint_as_float((x1 & k1) | (0xFF800000u & ~k1)) - base);
-          rs += p0 + p1;
-          pk[e >> 1] = pack_bf16x2(p0, p1);
-        }
-#pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2) {
-          const int ch = g4 * 2 + h2;
-          const uint32_t addr = prow + (((ch ^ row) & 7) << 4);
-          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(pk[h2 * 4 + 0]),
-                       "r"(pk[h2 * 4 + 1]), "r"(pk[h2 * 4 + 2]), "r"(pk[h2 * 4 + 3])
-                       : "memory");
+        for (int bk = 0; bk < 8; ++bk) {
+          asm volatile("st.shared.b32 [%0], %1;\n" ::"r"(rowa + (((bk ^ ra) & 7) << 4)), "r"(pa[bk]) : "memory");
+          asm volatile("st.shared.b32 [%0], %1;\n" ::"r"(rowb + (((bk ^ rb) & 7) << 4)), "r"(pb[bk]) : "memory");
         }
       }
-      l_sum = l_sum * alpha + rs;
-      sm100::tc_fence_before();
-      __syncwarp();
-      if (lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.s_free[sb]));
       sm100::fence_proxy_async_smem();
-      // Raise O to the new maximum (rare): needs the previous PV product done.
-      if (j > 0 && __any_sync(adt::kFullMask, need)) {
+      // Raise O to the new maxima (rare): needs the previous PV product done.
+      if (j > 0 && __any_sync(adt::kFullMask, needa || needb)) {
         if (!__all_sync(adt::kFullMask,
                         wait_bar(&bars.pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, &s_abort, p.err)))
           break;
         sm100::tc_fence_after();
 #pragma unroll 1
-        for (int c0 = 0; c0 < D; c0 += 16) {
-          uint32_t o[16];
-          sm100::tmem_ld16(tmem + lane_base + kOCol + c0, o);
+        for (int c0 = 0; c0 < D; c0 += 64) {
+          uint32_t o[32];
+          tmem_ld_16x256b_x8(tmem + lane_base + kOCol + c0, o);
           sm100::tmem_wait_ld();
 #pragma unroll
-          for (int e = 0; e < 16; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-          sm100::tmem_st16(tmem + lane_base + kOCol + c0, o);
+          for (int bk = 0; bk < 8; ++bk) {
+            o[4 * bk + 0] = __float_as_uint(__uint_as_float(o[4 * bk + 0]) * alpha_a);
+            o[4 * bk + 1] = __float_as_uint(__uint_as_float(o[4 * bk + 1]) * alpha_a);
+            o[4 * bk + 2] = __float_as_uint(__uint_as_float(o[4 * bk + 2]) * alpha_b);
+            o[4 * bk + 3] = __float_as_uint(__uint_as_float(o[4 * bk + 3]) * alpha_b);
+          }
+          tmem_st_16x256b_x8(tmem + lane_base + kOCol + c0, o);
         }
         sm100::tmem_wait_st();
       }
-      m_used = new_m;
+      mua = nma;
+      mub = nmb;
       sm100::tc_fence_before();
       __syncwarp();
       if (lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.p_full[sb]));
     }
+    // Full row sums: add the four shares of each quad.
+    la += __shfl_xor_sync(adt::kFullMask, la, 1);
+    la += __shfl_xor_sync(adt::kFullMask, la, 2);
+    lb += __shfl_xor_sync(adt::kFullMask, lb, 1);
+    lb += __shfl_xor_sync(adt::kFullMask, lb, 2);
+    m_ra = mua;
+    l_ra = la;
+    m_rb = mub;
+    l_rb = lb;
   }
 
   // ------------------------------------------------------------ epilogue
@@ -451,30 +512,41 @@ __global__ void __launch_bounds__(kThreads, 1)
   float2* sml = reinterpret_cast<float2*>(sStage + kMaxNodes * MS * 4);  // [64]
   float* sw = reinterpret_cast<float*>(sStage + kMaxNodes * MS * 4 + kMaxNodes * 8);  // weights
   if (warp < kSoftmaxWarps) {
+    const int g8 = lane >> 2, t4 = lane & 3;
+    const int ra = warp * 16 + g8, rb = ra + 8;
     // A split without key units (kv_len shorter than max_kv) contributes
     // nothing: weight 0, zero partial.
     const bool ok = nu > 0 && !s_abort && __all_sync(adt::kFullMask, wait_bar(&bars.o_full, 0, &s_abort, p.err));
-    if (!ok && lane < 16 && row < n) {
-      for (int c = 0; c < D; c += 4) *reinterpret_cast<float4*>(so + row * MS + c) = make_float4(0.f, 0.f, 0.f, 0.f);
-      sml[row] = make_float2(-INFINITY, 0.f);
-    }
     if (ok) {
       sm100::tc_fence_after();
       const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
-#pragma unroll
-      for (int c0 = 0; c0 < D; c0 += 16) {
-        uint32_t o[16];
-        sm100::tmem_ld16(tmem + lane_base + kOCol + c0, o);
+#pragma unroll 1
+      for (int c0 = 0; c0 < D; c0 += 64) {
+        uint32_t o[32];
+        tmem_ld_16x256b_x8(tmem + lane_base + kOCol + c0, o);
         sm100::tmem_wait_ld();
-        if (lane < 16 && row < n) {
 #pragma unroll
-          for (int e = 0; e < 16; e += 4)
-            *reinterpret_cast<float4*>(so + row * MS + c0 + e) =
-                make_float4(__uint_as_float(o[e]), __uint_as_float(o[e + 1]), __uint_as_float(o[e + 2]),
-                            __uint_as_float(o[e + 3]));
+        for (int bk = 0; bk < 8; ++bk) {
+          const int c = c0 + 8 * bk + 2 * t4;
+          if (ra < n)
+            *reinterpret_cast<float2*>(so + ra * MS + c) = make_float2(__uint_as_float(o[4 * bk]), __uint_as_float(o[4 * bk + 1]));
+          if (rb < n)
+            *reinterpret_cast<float2*>(so + rb * MS + c) =
+                make_float2(__uint_as_float(o[4 * bk + 2]), __uint_as_float(o[4 * bk + 3]));
         }
       }
-      if (lane < 16 && row < n) sml[row] = make_float2(m_used, l_sum);
+      if (t4 == 0) {
+        if (ra < n) sml[ra] = make_float2(m_ra, l_ra);
+        if (rb < n) sml[rb] = make_float2(m_rb, l_rb);
+      }
+    } else if (t4 == 0) {
+      for (int half = 0; half < 2; ++half) {
+        const int rr = half ? rb : ra;
+        if (rr < n) {
+          for (int c = 0; c < D; c += 4) *reinterpret_cast<float4*>(so + rr * MS + c) = make_float4(0.f, 0.f, 0.f, 0.f);
+          sml[rr] = make_float2(-INFINITY, 0.f);
+        }
+      }
     }
   }
   sm100::tc_fence_before();
@@ -508,15 +580,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int idx = tid; idx < rows_mine * kC4; idx += kThreads) {
       const int i = idx / kC4, c4 = idx % kC4;
       const int rr = rank + S * i;
+      // Issue every peer's load before combining (latency, not bandwidth, bound).
+      float4 v[kMaxClusterSplits];
+#pragma unroll
+      for (int c = 0; c < kMaxClusterSplits; ++c) {
+        v[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (c < S && sw[i * S + c] != 0.f)
+          v[c] = *reinterpret_cast<const float4*>(cl.map_shared_rank(so, c) + rr * MS + c4 * 4);
+      }
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int c = 0; c < S; ++c) {
-        const float w = sw[i * S + c];
-        if (w == 0.f) continue;
-        const float4 v = *reinterpret_cast<const float4*>(cl.map_shared_rank(so, c) + rr * MS + c4 * 4);
-        acc.x += w * v.x;
-        acc.y += w * v.y;
-        acc.z += w * v.z;
-        acc.w += w * v.w;
+#pragma unroll
+      for (int c = 0; c < kMaxClusterSplits; ++c) {
+        const float w = c < S ? sw[i * S + c] : 0.f;
+        acc.x += w * v[c].x;
+        acc.y += w * v[c].y;
+        acc.z += w * v[c].z;
+        acc.w += w * v[c].w;
       }
       __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + rr) * p.H + h) * D + c4 * 4;
       uint2 pk;
