@@ -7,26 +7,32 @@
 // tree sees are cut into units of 64: ceil(L/64) prefix units plus one tree
 // unit (its <= 64 nodes, masked per query row by an ancestor bitmask built
 // from the parent pointers).  Grid = (splits, H, B), one CTA per SM; a CTA
-// handles one (tree, head) and a contiguous share of the units.
+// handles one (tree, head) and a contiguous share of the units, which it
+// walks in chunks: the tree unit first (its K/V are loaded with Q), then the
+// prefix units two at a time (128 keys).
 //
-// Warp roles inside a CTA (192 threads):
-//   warp 4    producer: TMA tensor loads of prefix K/V chunks (128-byte
-//             swizzle) into a ring of stages; the tree unit (rows of
-//             k_tree / v_tree that TMA cannot bound) with cp.async;
-//   warp 5    one elected thread issues tcgen05.mma: S = Q K^T into a
-//             double-buffered tensor-memory tile (M = 64 queries, N = 64
-//             keys), then O += P V (N = head_dim, V read MN-major);
+// Warp roles inside a CTA (256 threads; one thread of each of warps 4-7):
+//   warp 4    TMA tensor loads of prefix K (64 x 64 boxes, 128-byte swizzle)
+//             into a ring of 128-key stages;
+//   warp 5    tcgen05.mma S = Q K^T into one of two tensor-memory tiles
+//             (M = 64 queries, N = 128 keys); frees the K tile once S is done;
+//   warp 6    TMA loads of prefix V into the same stages;
+//   warp 7    tcgen05.mma O += P V (N = head_dim, V read MN-major);
 //   warps 0-3 softmax: warp w owns query rows 16w .. 16w+15 (tensor-memory
 //             lanes 32w .. 32w+15 for M = 64), read with the 16x256b shape so
-//             that each thread holds two rows x 16 columns of a chunk; masks
-//             branch-free, exponentiates against a lazily raised running
-//             maximum (O is rescaled only when a row maximum grows by more
-//             than 2^8), writes P (bf16) to shared memory for the PV
-//             product; at the end they read O and l and emit the partial.
-// mbarriers connect the roles; every wait is bounded and a timeout sets
-// ADT_DEVERR_TIMEOUT.  The splits of one (tree, head) form a thread-block
-// cluster (<= 8) and merge their partials through distributed shared
-// memory; with more splits they merge through the workspace.
+//             that each thread holds two rows; exponentiates against a lazily
+//             raised running maximum (O is rescaled only when a row maximum
+//             grows by more than 2^8), writes P (bf16) with stmatrix for the
+//             PV product, and at the end reads O and l for the merge.
+// K and V of a stage are released separately (K when S is done, V and the P
+// buffer when PV is done), and S and PV are issued by different threads, so
+// loads of later chunks never queue behind the softmax of earlier ones.
+// Every mbarrier wait is bounded; a timeout sets ADT_DEVERR_TIMEOUT.
+//
+// The splits of one (tree, head) form a thread-block cluster (<= 8).  Each
+// split pushes its unnormalised partial rows (O, running max, row sum) into
+// the shared memory of the split that owns those rows, which then merges
+// them locally; with more splits they merge through the workspace.
 #include <cooperative_groups.h>
 #include <cuda.h>
 
@@ -39,37 +45,46 @@ namespace cg = cooperative_groups;
 
 namespace {
 
-constexpr int kUnit = 64;               // keys per pipeline unit
+constexpr int kUnit = 64;               // keys per split unit; the tree unit
+constexpr int kChunk = 128;             // keys per pipeline chunk
 constexpr int kMaxNodes = 64;           // tree nodes (query rows) per (tree, head)
 constexpr int kSoftmaxWarps = 4;
-constexpr int kProducerWarp = 4;
-constexpr int kMmaWarp = 5;
-constexpr int kThreads = 6 * 32;
+constexpr int kKLoadWarp = 4;
+constexpr int kSMmaWarp = 5;
+constexpr int kVLoadWarp = 6;
+constexpr int kPvMmaWarp = 7;
+constexpr int kThreads = 8 * 32;
 constexpr int kMaxClusterSplits = 8;    // portable cluster size
 constexpr int kMaxSplits = 96;          // workspace merge: weights fit in shared memory
-constexpr int kMaxStages = 8;
+constexpr int kMaxStages = 4;
 constexpr uint32_t kWaitLimit = 1u << 20;
-constexpr uint32_t kTmemCols = 256;     // S double buffer (2 x 64 columns) + O (<= 128 columns)
-constexpr uint32_t kOCol = 128;
+constexpr uint32_t kTmemCols = 512;     // two S tiles of 128 columns, then O (<= 128 columns)
+constexpr uint32_t kSCols = 128;
+constexpr uint32_t kOCol = 256;
 constexpr float kLn2 = 0.69314718055994530942f;
 constexpr float kLog2e = 1.44269504088896340736f;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 template <int D>
 struct Cfg {
-  static constexpr int kBlocks = D / 64;             // 128-byte column blocks per row
-  static constexpr int kBlockBytes = kUnit * 128;    // one column block of 64 rows
-  static constexpr int kTileBytes = kBlocks * kBlockBytes;  // 64 rows x D bf16
-  static constexpr int kStages = D == 128 ? 4 : 8;
+  static constexpr int kBlocks = D / 64;                 // 128-byte column blocks per row
+  static constexpr int kBlock64 = kUnit * 128;           // one column block of 64 rows
+  static constexpr int kBlock128 = kChunk * 128;         // one column block of 128 rows
+  static constexpr int kTreeTile = kBlocks * kBlock64;   // 64 rows x D
+  static constexpr int kStageTile = kBlocks * kBlock128; // 128 rows x D
+  static constexpr int kStageBytes = 2 * kStageTile;     // K tile, then V tile
+  static constexpr int kPBytes = 2 * kBlock64;           // 64 query rows x 128 keys
+  static constexpr int kStages = D == 128 ? 2 : 4;
   static constexpr int kQOff = 0;
-  static constexpr int kPOff = kTileBytes;                  // two P buffers (64 x 64 bf16)
-  static constexpr int kTreeOff = kPOff + 2 * kBlockBytes;    // tree unit: K tile, then V tile
-  static constexpr int kStageOff = kTreeOff + 2 * kTileBytes;
-  static constexpr int kStageBytes = 2 * kTileBytes;        // K tile, then V tile
+  static constexpr int kPOff = kTreeTile;                // Q is 64 rows x D, like a tree tile
+  static constexpr int kTreeOff = kPOff + 2 * kPBytes;   // tree unit: K tile, then V tile
+  static constexpr int kStageOff = kTreeOff + 2 * kTreeTile;
   static constexpr int kDynSmem = kStageOff + kStages * kStageBytes + 1024;  // + alignment slack
-  static constexpr uint32_t kIdescS = sm100::idesc_bf16_f32(64, 64, 0, 0);
+  static constexpr uint32_t kIdescS128 = sm100::idesc_bf16_f32(64, 128, 0, 0);
+  static constexpr uint32_t kIdescS64 = sm100::idesc_bf16_f32(64, 64, 0, 0);
   static constexpr uint32_t kIdescO = sm100::idesc_bf16_f32(64, D, 0, 1);
-  static constexpr int kMergeStride = D + 4;                // fp32 per row of a parked partial
+  static constexpr int kSlotStride = D + 8;  // fp32 per pushed row: conflict-free float2 stores
+  static_assert(kStages <= kMaxStages, "stage ring");
 };
 
 struct TcParams {
@@ -90,8 +105,9 @@ struct TcParams {
   unsigned* err;
 };
 
-// Byte offset of 16-byte chunk `ch` (0 .. D/8-1) of row `row` in a tile of
-// 128-byte column blocks with the 128-byte swizzle (the layout TMA writes).
+// Byte offset of 16-byte chunk `ch` (0 .. D/8-1) of row `row` in a 64-row
+// tile of 128-byte column blocks with the 128-byte swizzle (the layout TMA
+// writes).
 __device__ __forceinline__ uint32_t sw128_off(int row, int ch) {
   return static_cast<uint32_t>((ch >> 3) * (kUnit * 128) + row * 128 + (((ch & 7) ^ (row & 7)) << 4));
 }
@@ -99,13 +115,34 @@ __device__ __forceinline__ uint32_t sw128_off(int row, int ch) {
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
 }
+__device__ __forceinline__ void cp_async4(uint32_t dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(dst), "l"(src) : "memory");
+}
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;\n" ::: "memory"); }
+
+// Named barrier over the four softmax warps.
+__device__ __forceinline__ void softmax_warps_sync() { asm volatile("bar.sync 1, 128;\n" ::: "memory"); }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// 2^x with the hardware approximation (flush-to-zero); 2^-inf = 0.
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;\n" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Four 8x8 bf16 tiles to shared memory; thread l supplies the address of row
+// l % 8 of tile l / 8 and holds, in register i, row lane / 4, columns
+// 2 (lane % 4) .. +1 of tile i.
+__device__ __forceinline__ void stmatrix_x4(uint32_t addr, uint32_t r0, uint32_t r1, uint32_t r2, uint32_t r3) {
+  asm volatile("stmatrix.sync.aligned.m8n8.x4.shared.b16 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(r0), "r"(r1),
+               "r"(r2), "r"(r3)
+               : "memory");
+}
 
 // tcgen05.ld / st, shape 16x256b, 8 repetitions: for an M = 64 accumulator
 // (rows 16w .. 16w+15 in lanes 32w .. 32w+15), thread (g = lane / 4,
@@ -134,21 +171,82 @@ __device__ __forceinline__ void tmem_st_16x256b_x8(uint32_t taddr, const uint32_
       : "memory");
 }
 
-// x masked to -inf where the keep bit is 0, without branching.
+// x masked to -inf where the keep bit is 0, without branching (a NaN score
+// at a masked position also becomes -inf).
 __device__ __forceinline__ float mask_or_neg_inf(float x, uint32_t keep_bit) {
   const uint32_t keep = 0u - keep_bit;
   return __uint_as_float((__float_as_uint(x) & keep) | (0xFF800000u & ~keep));
 }
 
+// Softmax of one chunk for the two rows (a, b) a thread holds: NB 8-column
+// blocks (8 for 64 keys, 16 for 128), scores in sa / sb (raw Q.K), keep
+// masks (bit c = column c) applied only when `masked`.  Updates the lazily
+// raised maxima mu (log2 units), the row-sum shares l, returns the rescale
+// factors of O and the bf16 probabilities packed in column pairs.
+template <int NB>
+__device__ __forceinline__ void chunk_softmax(float (&sa)[32], float (&sb)[32], bool masked, uint64_t ka0,
+                                              uint64_t ka1, uint64_t kb0, uint64_t kb1, int t4, float scale,
+                                              float& mu_a, float& mu_b, float& l_a, float& l_b, float& alpha_a,
+                                              float& alpha_b, uint32_t (&pa)[16], uint32_t (&pb)[16]) {
+  if (masked) {
+    const int sh = 2 * t4;
+    const uint64_t a0 = ka0 >> sh, a1 = ka1 >> sh, b0 = kb0 >> sh, b1 = kb1 >> sh;
+#pragma unroll
+    for (int bk = 0; bk < NB; ++bk) {
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int c = 8 * (bk & 7) + e;
+        const uint64_t ma = bk < 8 ? a0 : a1, mb = bk < 8 ? b0 : b1;
+        sa[2 * bk + e] = mask_or_neg_inf(sa[2 * bk + e], static_cast<uint32_t>(ma >> c) & 1u);
+        sb[2 * bk + e] = mask_or_neg_inf(sb[2 * bk + e], static_cast<uint32_t>(mb >> c) & 1u);
+      }
+    }
+  }
+  float mxa = sa[0], mxb = sb[0];
+#pragma unroll
+  for (int i = 1; i < 2 * NB; ++i) {
+    mxa = fmaxf(mxa, sa[i]);
+    mxb = fmaxf(mxb, sb[i]);
+  }
+  mxa = fmaxf(mxa, __shfl_xor_sync(adt::kFullMask, mxa, 1));
+  mxa = fmaxf(mxa, __shfl_xor_sync(adt::kFullMask, mxa, 2));
+  mxb = fmaxf(mxb, __shfl_xor_sync(adt::kFullMask, mxb, 1));
+  mxb = fmaxf(mxb, __shfl_xor_sync(adt::kFullMask, mxb, 2));
+  mxa *= scale;  // scale > 0: the maximum of the scaled scores
+  mxb *= scale;
+  const bool needa = mxa > mu_a + kRescaleThreshold, needb = mxb > mu_b + kRescaleThreshold;
+  const float nma = needa ? mxa : mu_a, nmb = needb ? mxb : mu_b;
+  alpha_a = needa ? ex2_approx(mu_a - nma) : 1.f;
+  alpha_b = needb ? ex2_approx(mu_b - nmb) : 1.f;
+  const float base_a = nma == -INFINITY ? 0.f : nma, base_b = nmb == -INFINITY ? 0.f : nmb;
+  float ra[4] = {0.f, 0.f, 0.f, 0.f}, rb[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int bk = 0; bk < NB; ++bk) {
+    const float a0 = ex2_approx(fmaf(sa[2 * bk], scale, -base_a));
+    const float a1 = ex2_approx(fmaf(sa[2 * bk + 1], scale, -base_a));
+    const float b0 = ex2_approx(fmaf(sb[2 * bk], scale, -base_b));
+    const float b1 = ex2_approx(fmaf(sb[2 * bk + 1], scale, -base_b));
+    ra[bk & 3] += a0 + a1;
+    rb[bk & 3] += b0 + b1;
+    pa[bk] = pack_bf16x2(a0, a1);
+    pb[bk] = pack_bf16x2(b0, b1);
+  }
+  l_a = l_a * alpha_a + ((ra[0] + ra[1]) + (ra[2] + ra[3]));
+  l_b = l_b * alpha_b + ((rb[0] + rb[1]) + (rb[2] + rb[3]));
+  mu_a = nma;
+  mu_b = nmb;
+}
+
 struct Barriers {
-  uint64_t q_full;
-  uint64_t kv_full[kMaxStages];
-  uint64_t kv_empty[kMaxStages];
+  uint64_t q_full;                 // Q and the tree unit's K/V are in shared memory
+  uint64_t k_full[kMaxStages];     // a stage's K tile has landed
+  uint64_t v_full[kMaxStages];     // a stage's V tile has landed
+  uint64_t k_free[kMaxStages];     // the S product of the chunk in that slot finished
+  uint64_t done[kMaxStages];       // the PV product of the chunk in that slot finished
   uint64_t s_full[2];
   uint64_t s_free[2];
   uint64_t p_full[2];
-  uint64_t pv_done[2];
-  uint64_t o_full;
+  uint64_t drain[2];               // abort path: every MMA a thread issued finished
 };
 
 // Bounded wait that also gives up when another role has aborted.
@@ -173,6 +271,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   __shared__ Barriers bars;
   __shared__ uint64_t anc[kMaxNodes];
+  __shared__ int s_par[kMaxNodes];
+  __shared__ float s_w[kMaxNodes + kMaxClusterSplits];
   __shared__ uint32_t tmem_slot;
   __shared__ int s_bad;
   __shared__ int s_last;
@@ -184,49 +284,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int node0 = p.offs[b];
   const int n = p.offs[b + 1] - node0;
+  const int total_nodes = p.offs[p.B];
   const int L = p.kv_len[b];
 
-  if (tid == 0) {
-    s_bad = 0;
-    s_abort = 0;
-  }
-  __syncthreads();
   // Conditions that hold for every CTA of this (tree, head): all leave here.
-  if (n < 1 || n > kMaxNodes) {
+  if (n < 1 || n > kMaxNodes || node0 < 0 || node0 + n > total_nodes) {
     if (split == 0 && h == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_BAD_TREE);
     return;
   }
   if (L < 0 || L > p.max_kv) {
     if (split == 0 && h == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_KV_RANGE);
-    return;
-  }
-  // Ancestor bitmask of every node: bit j of anc[t] <=> j in ans(t) or j == t.
-  if (tid < kMaxNodes) {
-    uint64_t m = 0;
-    if (tid < n) {
-      int j = tid;
-      int par = p.parents[node0 + j];
-      m = 1ull << j;
-      if ((j == 0) != (par < 0)) s_bad = 1;
-      while (par >= 0) {
-        if (par >= j) {
-          s_bad = 1;
-          break;
-        }
-        m |= 1ull << par;
-        j = par;
-        par = p.parents[node0 + j];
-        if ((j == 0) != (par < 0)) {
-          s_bad = 1;
-          break;
-        }
-      }
-    }
-    anc[tid] = m;
-  }
-  __syncthreads();
-  if (s_bad) {
-    if (split == 0 && h == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_BAD_TREE);
     return;
   }
 
@@ -235,13 +302,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int u_begin = static_cast<int>(static_cast<int64_t>(split) * U / S);
   const int u_end = static_cast<int>(static_cast<int64_t>(split + 1) * U / S);
   const int nu = u_end - u_begin;
-  // The CTA whose share ends with the tree unit processes it first (its K/V
-  // are loaded with Q at the start); prefix units follow in order through
-  // the TMA ring.  Iteration j handles unit unit_of(j).
+  // Chunk 0 is the tree unit for the CTA whose share ends with it; prefix
+  // units follow two per chunk (the last chunk may hold one).
   const int has_tree = (u_end == U && nu > 0) ? 1 : 0;
   const int np = nu - has_tree;  // prefix units of this CTA
-  auto unit_of = [&](int j) { return has_tree ? (j == 0 ? U - 1 : u_begin + j - 1) : u_begin + j; };
+  const int nch = has_tree + (np + 1) / 2;
   const int NS = C::kStages;
+  auto chunk_keys = [&](int j) -> int {
+    if (has_tree && j == 0) return kUnit;
+    const int pc = j - has_tree;
+    return (np - 2 * pc >= 2 ? 2 : 1) * kUnit;
+  };
+  auto chunk_key0 = [&](int j) -> int { return (u_begin + 2 * (j - has_tree)) * kUnit; };
 
   uint8_t* sQ = smem + C::kQOff;
   uint8_t* sP = smem + C::kPOff;
@@ -249,130 +321,206 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* sTree = smem + C::kTreeOff;
 
   if (tid == 0) {
+    s_bad = 0;
+    s_abort = 0;
     sm100::mbar_init(sm100::smem_addr(&bars.q_full), kSoftmaxWarps);
     for (int s = 0; s < NS; ++s) {
-      sm100::mbar_init(sm100::smem_addr(&bars.kv_full[s]), 1);
-      sm100::mbar_init(sm100::smem_addr(&bars.kv_empty[s]), 1);
+      sm100::mbar_init(sm100::smem_addr(&bars.k_full[s]), 1);
+      sm100::mbar_init(sm100::smem_addr(&bars.v_full[s]), 1);
+      sm100::mbar_init(sm100::smem_addr(&bars.k_free[s]), 1);
+      sm100::mbar_init(sm100::smem_addr(&bars.done[s]), 1);
     }
     for (int s = 0; s < 2; ++s) {
       sm100::mbar_init(sm100::smem_addr(&bars.s_full[s]), 1);
       sm100::mbar_init(sm100::smem_addr(&bars.s_free[s]), kSoftmaxWarps);
       sm100::mbar_init(sm100::smem_addr(&bars.p_full[s]), kSoftmaxWarps);
-      sm100::mbar_init(sm100::smem_addr(&bars.pv_done[s]), 1);
     }
-    sm100::mbar_init(sm100::smem_addr(&bars.o_full), 1);
+    sm100::mbar_init(sm100::smem_addr(&bars.drain[0]), 1);
+    sm100::mbar_init(sm100::smem_addr(&bars.drain[1]), 1);
     sm100::fence_mbar_init();
   }
   if (warp == 0) {
     sm100::tmem_alloc(sm100::smem_addr(&tmem_slot), kTmemCols);
     sm100::tmem_relinquish();
   }
+  if (warp < kSoftmaxWarps) {
+    // Q tile: rows node0 .. node0+63 (rows past the tree zero-filled); the
+    // tree unit's K/V for kv head g likewise; the parent pointers.
+    for (int i = tid; i < kUnit * (D / 8); i += kSoftmaxWarps * 32) {
+      const int r = i / (D / 8), ch = i % (D / 8);
+      const bool valid = r < n;
+      const int row = node0 + (valid ? r : 0);
+      cp_async16(sm100::smem_addr(sQ) + sw128_off(r, ch), p.q + (static_cast<int64_t>(row) * p.H + h) * D + ch * 8,
+                 valid ? 16 : 0);
+      if (has_tree) {
+        const int64_t off = (static_cast<int64_t>(row) * p.Hkv + g) * D + ch * 8;
+        cp_async16(sm100::smem_addr(sTree) + sw128_off(r, ch), p.kt + off, valid ? 16 : 0);
+        cp_async16(sm100::smem_addr(sTree + C::kTreeTile) + sw128_off(r, ch), p.vt + off, valid ? 16 : 0);
+      }
+    }
+    if (tid < n) cp_async4(sm100::smem_addr(&s_par[tid]), p.parents + node0 + tid);
+  }
   sm100::tc_fence_before();
   __syncthreads();
   sm100::tc_fence_after();
   const uint32_t tmem = tmem_slot;
 
+  // Stage loads: chunk j goes to slot j % NS, K tile by warp 4 and V tile by
+  // warp 6.  The tree chunk loads nothing (its K/V came with Q) but still
+  // completes its slot's phases, so that every slot's phases advance once
+  // per chunk.
+  const bool is_loader = (warp == kKLoadWarp || warp == kVLoadWarp) && lane == 0;
+  const bool load_v = warp == kVLoadWarp;
+  auto issue_tile = [&](int j) {
+    const int st = j % NS;
+    const uint32_t bar = sm100::smem_addr(load_v ? &bars.v_full[st] : &bars.k_full[st]);
+    if (has_tree && j == 0) {
+      sm100::mbar_arrive(bar);
+      return;
+    }
+    const int halves = chunk_keys(j) / kUnit;
+    const int key0 = chunk_key0(j);
+    uint8_t* dst = sStage + st * C::kStageBytes + (load_v ? C::kStageTile : 0);
+    const CUtensorMap* map = load_v ? &tm_v : &tm_k;
+    sm100::mbar_arrive_expect_tx(bar, C::kBlocks * halves * C::kBlock64);
+    for (int blk = 0; blk < C::kBlocks; ++blk) {
+      for (int hf = 0; hf < halves; ++hf)
+        sm100::tma_load_4d(sm100::smem_addr(dst + blk * C::kBlock128 + hf * C::kBlock64), map, blk * 64,
+                           key0 + hf * kUnit, g, b, bar);
+    }
+  };
+  const int first_issue = nch < NS ? nch : NS;
+  if (is_loader) {
+    for (int j = 0; j < first_issue; ++j) issue_tile(j);
+  }
+  if (warp < kSoftmaxWarps) {
+    cp_async_wait_all();
+    softmax_warps_sync();
+    // Ancestor bitmask of every node: bit j of anc[t] <=> j in ans(t) or j == t.
+    if (tid < kMaxNodes) {
+      uint64_t m = 0;
+      if (tid < n) {
+        int j = tid;
+        int par = s_par[j];
+        m = 1ull << j;
+        bool bad = (j == 0) != (par < 0);
+        while (!bad && par >= 0) {
+          if (par >= j) {
+            bad = true;
+            break;
+          }
+          m |= 1ull << par;
+          j = par;
+          par = s_par[j];
+          bad = (j == 0) != (par < 0);
+        }
+        if (bad) s_bad = 1;
+      }
+      anc[tid] = m;
+    }
+  }
+  __syncthreads();
+  if (s_bad) {
+    // Same tree for every CTA of the cluster: all leave here, after the
+    // loads already issued have landed.
+    if (split == 0 && h == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_BAD_TREE);
+    if (is_loader) {
+      for (int j = 0; j < first_issue; ++j)
+        (void)sm100::mbar_wait_bounded(sm100::smem_addr(load_v ? &bars.v_full[j % NS] : &bars.k_full[j % NS]), 0,
+                                       kWaitLimit);
+    }
+    sm100::tc_fence_before();
+    __syncthreads();
+    if (warp == 0) sm100::tmem_dealloc(tmem, kTmemCols);
+    return;
+  }
+
   // Final row statistics of the softmax threads' two rows (a, b).
   float m_ra = -INFINITY, l_ra = 0.f, m_rb = -INFINITY, l_rb = 0.f;
 
-  if (warp == kProducerWarp) {
-    // ------------------------------------------------------------ producer
-    int issued = 0;
-    for (int jp = 0; jp < np; ++jp) {
-      const int st = jp % NS;
-      if (jp >= NS &&
-          !__all_sync(adt::kFullMask, wait_bar(&bars.kv_empty[st], ((jp / NS) - 1) & 1, &s_abort, p.err)))
-        break;
-      if (lane == 0) {
-        uint8_t* kdst = sStage + st * C::kStageBytes;
-        uint8_t* vdst = kdst + C::kTileBytes;
-        const uint32_t bar = sm100::smem_addr(&bars.kv_full[st]);
-        sm100::mbar_arrive_expect_tx(bar, 2 * C::kTileBytes);
-        const int key0 = (u_begin + jp) * kUnit;
-        for (int blk = 0; blk < C::kBlocks; ++blk) {
-          sm100::tma_load_4d(sm100::smem_addr(kdst + blk * C::kBlockBytes), &tm_k, blk * 64, key0, g, b, bar);
-          sm100::tma_load_4d(sm100::smem_addr(vdst + blk * C::kBlockBytes), &tm_v, blk * 64, key0, g, b, bar);
-        }
+  if (warp == kKLoadWarp || warp == kVLoadWarp) {
+    // ------------------------------------------------------------ K / V loads
+    if (lane == 0) {
+      int issued = first_issue;
+      for (int j = first_issue; j < nch; ++j) {
+        const int st = j % NS;
+        // slot st was last used by chunk j - NS: its K is free once its S is
+        // done, its V once its PV is done
+        if (!wait_bar(load_v ? &bars.done[st] : &bars.k_free[st], ((j / NS) - 1) & 1, &s_abort, p.err)) break;
+        issue_tile(j);
+        ++issued;
       }
-      __syncwarp();
-      ++issued;
+      if (s_abort) {
+        // let every copy still in flight land before the CTA can exit
+        for (int j = (issued > NS ? issued - NS : 0); j < issued; ++j)
+          (void)sm100::mbar_wait_bounded(sm100::smem_addr(load_v ? &bars.v_full[j % NS] : &bars.k_full[j % NS]),
+                                         (j / NS) & 1, kWaitLimit);
+      }
     }
-    if (s_abort && lane == 0) {
-      // let every copy still in flight land before the CTA can exit
-      for (int jp = (issued > NS ? issued - NS : 0); jp < issued; ++jp)
-        (void)sm100::mbar_wait_bounded(sm100::smem_addr(&bars.kv_full[jp % NS]), (jp / NS) & 1, kWaitLimit);
-    }
-  } else if (warp == kMmaWarp) {
-    // ------------------------------------------------------------ MMA issuer
+    __syncwarp();
+  } else if (warp == kSMmaWarp) {
+    // ------------------------------------------------------------ S = Q K^T
     if (lane == 0) {
       bool ok = wait_bar(&bars.q_full, 0, &s_abort, p.err);
       const uint32_t q_addr = sm100::smem_addr(sQ);
-      const uint32_t p_addr = sm100::smem_addr(sP);
-      auto issue_pv = [&](int i) -> bool {
-        const int pb = i & 1;
-        if (!wait_bar(&bars.p_full[pb], (i >> 1) & 1, &s_abort, p.err)) return false;
+      for (int j = 0; ok && j < nch; ++j) {
+        const int st = j % NS, sb = j & 1;
+        if (!wait_bar(&bars.k_full[st], (j / NS) & 1, &s_abort, p.err) ||
+            (j >= 2 && !wait_bar(&bars.s_free[sb], ((j >> 1) - 1) & 1, &s_abort, p.err)))
+          break;
         sm100::tc_fence_after();
-        const bool tree_i = has_tree && i == 0;
-        const int ip = i - has_tree;
-        const uint32_t v_addr = tree_i ? sm100::smem_addr(sTree + C::kTileBytes)
-                                       : sm100::smem_addr(sStage + (ip % NS) * C::kStageBytes + C::kTileBytes);
-#pragma unroll
-        for (int kk = 0; kk < kUnit / 16; ++kk) {
-          const uint64_t da = sm100::smem_desc_sw128(p_addr + pb * C::kBlockBytes + kk * 32, 16, 1024);
-          const uint64_t db = sm100::smem_desc_sw128(v_addr + kk * 2048, C::kBlockBytes, 1024);
-          sm100::mma_bf16_ss(tmem + kOCol, da, db, C::kIdescO, (i > 0 || kk > 0) ? 1u : 0u);
-        }
-        if (!tree_i) sm100::mma_commit(sm100::smem_addr(&bars.kv_empty[ip % NS]));
-        sm100::mma_commit(sm100::smem_addr(&bars.pv_done[pb]));
-        return true;
-      };
-      for (int j = 0; ok && j < nu; ++j) {
         const bool tree_j = has_tree && j == 0;
-        const int jp = j - has_tree;
-        const int st = jp % NS, sb = j & 1;
-        if (!tree_j && !wait_bar(&bars.kv_full[st], (jp / NS) & 1, &s_abort, p.err)) break;
-        if (j >= 2 && !wait_bar(&bars.s_free[sb], ((j >> 1) - 1) & 1, &s_abort, p.err)) break;
-        sm100::tc_fence_after();
         const uint32_t k_addr = tree_j ? sm100::smem_addr(sTree) : sm100::smem_addr(sStage + st * C::kStageBytes);
+        const uint32_t k_blk = tree_j ? C::kBlock64 : C::kBlock128;
+        const uint32_t idesc = chunk_keys(j) == kChunk ? C::kIdescS128 : C::kIdescS64;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * C::kBlockBytes + (kk & 3) * 32;
-          const uint64_t da = sm100::smem_desc_sw128(q_addr + off, 16, 1024);
-          const uint64_t db = sm100::smem_desc_sw128(k_addr + off, 16, 1024);
-          sm100::mma_bf16_ss(tmem + sb * 64, da, db, C::kIdescS, kk > 0 ? 1u : 0u);
+          const uint64_t da = sm100::smem_desc_sw128(q_addr + (kk >> 2) * C::kBlock64 + (kk & 3) * 32, 16, 1024);
+          const uint64_t db = sm100::smem_desc_sw128(k_addr + (kk >> 2) * k_blk + (kk & 3) * 32, 16, 1024);
+          sm100::mma_bf16_ss(tmem + sb * kSCols, da, db, idesc, kk > 0 ? 1u : 0u);
         }
         sm100::mma_commit(sm100::smem_addr(&bars.s_full[sb]));
-        if (j >= 1 && !issue_pv(j - 1)) break;
-        if (j == nu - 1 && issue_pv(j)) sm100::mma_commit(sm100::smem_addr(&bars.o_full));
+        // Once S is done its K tile can be refilled.
+        if (!wait_bar(&bars.s_full[sb], (j >> 1) & 1, &s_abort, p.err)) break;
+        sm100::mbar_arrive(sm100::smem_addr(&bars.k_free[st]));
       }
       if (s_abort) {
         // wait for the tensor core to finish whatever was issued
-        sm100::mma_commit(sm100::smem_addr(&bars.o_full));
-        (void)sm100::mbar_wait_bounded(sm100::smem_addr(&bars.o_full), 0, kWaitLimit);
+        sm100::mma_commit(sm100::smem_addr(&bars.drain[0]));
+        (void)sm100::mbar_wait_bounded(sm100::smem_addr(&bars.drain[0]), 0, kWaitLimit);
+      }
+    }
+    __syncwarp();
+  } else if (warp == kPvMmaWarp) {
+    // ------------------------------------------------------------ O += P V
+    if (lane == 0) {
+      const uint32_t p_addr = sm100::smem_addr(sP);
+      for (int i = 0; i < nch; ++i) {
+        if (!wait_bar(&bars.p_full[i & 1], (i >> 1) & 1, &s_abort, p.err) ||
+            !wait_bar(&bars.v_full[i % NS], (i / NS) & 1, &s_abort, p.err))
+          break;
+        sm100::tc_fence_after();
+        const bool tree_i = has_tree && i == 0;
+        const uint32_t v_addr = tree_i ? sm100::smem_addr(sTree + C::kTreeTile)
+                                       : sm100::smem_addr(sStage + (i % NS) * C::kStageBytes + C::kStageTile);
+        const uint32_t v_lbo = tree_i ? C::kBlock64 : C::kBlock128;  // stride of V's d blocks
+        const uint32_t pb = p_addr + (i & 1) * C::kPBytes;
+        const int ksteps = chunk_keys(i) / 16;
+        for (int kk = 0; kk < ksteps; ++kk) {
+          const uint64_t da = sm100::smem_desc_sw128(pb + (kk >> 2) * C::kBlock64 + (kk & 3) * 32, 16, 1024);
+          const uint64_t db = sm100::smem_desc_sw128(v_addr + kk * 2048, v_lbo, 1024);
+          sm100::mma_bf16_ss(tmem + kOCol, da, db, C::kIdescO, (i > 0 || kk > 0) ? 1u : 0u);
+        }
+        sm100::mma_commit(sm100::smem_addr(&bars.done[i % NS]));
+      }
+      if (s_abort) {
+        sm100::mma_commit(sm100::smem_addr(&bars.drain[1]));
+        (void)sm100::mbar_wait_bounded(sm100::smem_addr(&bars.drain[1]), 0, kWaitLimit);
       }
     }
     __syncwarp();
   } else {
     // ------------------------------------------------------------ softmax warps 0-3
-    // Q tile: rows node0 .. node0+63 (rows past the tree zero-filled).
-    for (int i = tid; i < kUnit * (D / 8); i += kSoftmaxWarps * 32) {
-      const int r = i / (D / 8), ch = i % (D / 8);
-      const bool valid = r < n;
-      const __nv_bfloat16* src = p.q + (static_cast<int64_t>(node0 + (valid ? r : 0)) * p.H + h) * D + ch * 8;
-      cp_async16(sm100::smem_addr(sQ) + sw128_off(r, ch), src, valid ? 16 : 0);
-    }
-    if (has_tree) {
-      // Tree unit: rows node0 .. node0+63 of k_tree / v_tree for kv head g;
-      // rows past this tree are zero-filled, never read out of bounds.
-      for (int i = tid; i < kUnit * (D / 8); i += kSoftmaxWarps * 32) {
-        const int r = i / (D / 8), ch = i % (D / 8);
-        const bool valid = r < n;
-        const int64_t off = (static_cast<int64_t>(node0 + (valid ? r : 0)) * p.Hkv + g) * D + ch * 8;
-        cp_async16(sm100::smem_addr(sTree) + sw128_off(r, ch), p.kt + off, valid ? 16 : 0);
-        cp_async16(sm100::smem_addr(sTree + C::kTileBytes) + sw128_off(r, ch), p.vt + off, valid ? 16 : 0);
-      }
-    }
-    cp_async_wait_all();
     sm100::fence_proxy_async_smem();
     __syncwarp();
     if (lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.q_full));
@@ -386,89 +534,93 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint64_t ama = ra < n ? anc[ra] : 0ull;
     const uint64_t amb = rb < n ? anc[rb] : 0ull;
     const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
+    // stmatrix addressing: lane l writes row (l / 8 odd ? 8 : 0) + l % 8 of
+    // the warp's rows, in column block (l / 16) of each pair of blocks.
+    const int st_row = warp * 16 + ((lane >> 3) & 1) * 8 + (lane & 7);
+    const int st_blk = lane >> 4;
+    const float scale = p.scale_log2;
     float mua = -INFINITY, mub = -INFINITY;  // running maxima used for the exponentials
     float la = 0.f, lb = 0.f;                // this thread's share of the row sums
-    for (int j = 0; j < nu; ++j) {
+    for (int j = 0; j < nch; ++j) {
       const int sb = j & 1;
       if (!__all_sync(adt::kFullMask, wait_bar(&bars.s_full[sb], (j >> 1) & 1, &s_abort, p.err))) break;
       sm100::tc_fence_after();
-      uint32_t r[32];
-      tmem_ld_16x256b_x8(tmem + lane_base + sb * 64, r);
+      const int keys = chunk_keys(j);
+      uint32_t r0[32], r1[32];
+      tmem_ld_16x256b_x8(tmem + lane_base + sb * kSCols, r0);
+      if (keys == kChunk) tmem_ld_16x256b_x8(tmem + lane_base + sb * kSCols + 64, r1);
       sm100::tmem_wait_ld();
-      // S is in registers: hand the tensor-memory buffer back to the MMA warp.
+      // S is in registers: hand the tensor-memory tile back to the MMA warp.
       sm100::tc_fence_before();
       __syncwarp();
       if (lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.s_free[sb]));
 
-      const int u = unit_of(j);
-      // Which of the chunk's 64 keys a row sees (the prefix up to L, or the
-      // row's ancestors and itself in the tree unit), applied with bit
-      // operations so no lane branches on it.
-      uint64_t vma, vmb;
-      if (u == U - 1) {
-        vma = ama;
-        vmb = amb;
-      } else {
-        const int kl = L - u * kUnit;  // >= 1 for every prefix unit
-        vma = vmb = kl >= 64 ? ~0ull : ((1ull << kl) - 1ull);
+      // Which keys a row sees: its ancestors and itself in the tree unit,
+      // the prefix up to L otherwise.  Only the tree chunk and a chunk that
+      // holds the end of the prefix need a mask.
+      const bool tree_j = has_tree && j == 0;
+      const int kl = tree_j ? keys : L - chunk_key0(j);
+      const bool masked = tree_j || kl < keys;
+      uint64_t ka0 = ~0ull, ka1 = ~0ull, kb0 = ~0ull, kb1 = ~0ull;
+      if (tree_j) {
+        ka0 = ama;
+        kb0 = amb;
+      } else if (kl < keys) {
+        ka0 = kb0 = kl >= 64 ? ~0ull : ((1ull << kl) - 1ull);
+        ka1 = kb1 = kl >= 128 ? ~0ull : (kl > 64 ? ((1ull << (kl - 64)) - 1ull) : 0ull);
       }
-      const float scale = p.scale_log2;
-      float xa[16], xb[16];
-      float mxa = -INFINITY, mxb = -INFINITY;
+      float sa[32], sbv[32];
 #pragma unroll
       for (int bk = 0; bk < 8; ++bk) {
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const int c = 8 * bk + 2 * t4 + e;
-          xa[2 * bk + e] = mask_or_neg_inf(__uint_as_float(r[4 * bk + e]) * scale,
-                                           static_cast<uint32_t>(vma >> c) & 1u);
-          xb[2 * bk + e] = mask_or_neg_inf(__uint_as_float(r[4 * bk + 2 + e]) * scale,
-                                           static_cast<uint32_t>(vmb >> c) & 1u);
-          mxa = fmaxf(mxa, xa[2 * bk + e]);
-          mxb = fmaxf(mxb, xb[2 * bk + e]);
-        }
+        sa[2 * bk] = __uint_as_float(r0[4 * bk]);
+        sa[2 * bk + 1] = __uint_as_float(r0[4 * bk + 1]);
+        sbv[2 * bk] = __uint_as_float(r0[4 * bk + 2]);
+        sbv[2 * bk + 1] = __uint_as_float(r0[4 * bk + 3]);
+        sa[16 + 2 * bk] = __uint_as_float(r1[4 * bk]);
+        sa[16 + 2 * bk + 1] = __uint_as_float(r1[4 * bk + 1]);
+        sbv[16 + 2 * bk] = __uint_as_float(r1[4 * bk + 2]);
+        sbv[16 + 2 * bk + 1] = __uint_as_float(r1[4 * bk + 3]);
       }
-      mxa = fmaxf(mxa, __shfl_xor_sync(adt::kFullMask, mxa, 1));
-      mxa = fmaxf(mxa, __shfl_xor_sync(adt::kFullMask, mxa, 2));
-      mxb = fmaxf(mxb, __shfl_xor_sync(adt::kFullMask, mxb, 1));
-      mxb = fmaxf(mxb, __shfl_xor_sync(adt::kFullMask, mxb, 2));
-      // Lazily raised maximum: O is rescaled only when a row's maximum grows
-      // by more than 2^8 over the one its exponentials were taken against.
-      const bool needa = mxa > mua + kRescaleThreshold, needb = mxb > mub + kRescaleThreshold;
-      const float nma = needa ? mxa : mua, nmb = needb ? mxb : mub;
-      const float alpha_a = needa ? exp2f(mua - nma) : 1.f, alpha_b = needb ? exp2f(mub - nmb) : 1.f;
-      const float base_a = nma == -INFINITY ? 0.f : nma, base_b = nmb == -INFINITY ? 0.f : nmb;
-      float rsa = 0.f, rsb = 0.f;
-      uint32_t pa[8], pb[8];
-#pragma unroll
-      for (int bk = 0; bk < 8; ++bk) {
-        const float a0 = exp2f(xa[2 * bk] - base_a), a1 = exp2f(xa[2 * bk + 1] - base_a);
-        const float b0 = exp2f(xb[2 * bk] - base_b), b1 = exp2f(xb[2 * bk + 1] - base_b);
-        rsa += a0 + a1;
-        rsb += b0 + b1;
-        pa[bk] = pack_bf16x2(a0, a1);
-        pb[bk] = pack_bf16x2(b0, b1);
-      }
-      la = la * alpha_a + rsa;
-      lb = lb * alpha_b + rsb;
+      uint32_t pa[16], pb[16];
+      float alpha_a, alpha_b;
+      if (keys == kChunk)
+        chunk_softmax<16>(sa, sbv, masked, ka0, ka1, kb0, kb1, t4, scale, mua, mub, la, lb, alpha_a, alpha_b, pa, pb);
+      else
+        chunk_softmax<8>(sa, sbv, masked, ka0, ka1, kb0, kb1, t4, scale, mua, mub, la, lb, alpha_a, alpha_b, pa, pb);
+
       // P buffer sb was last read by the PV product of chunk j - 2.
-      if (j >= 2 &&
-          !__all_sync(adt::kFullMask, wait_bar(&bars.pv_done[sb], ((j >> 1) - 1) & 1, &s_abort, p.err)))
+      if (j >= 2 && !__all_sync(adt::kFullMask,
+                                wait_bar(&bars.done[(j - 2) % NS], ((j - 2) / NS) & 1, &s_abort, p.err)))
         break;
       {
-        const uint32_t pbase = sm100::smem_addr(sP + sb * C::kBlockBytes);
-        const uint32_t rowa = pbase + ra * 128 + t4 * 4, rowb = pbase + rb * 128 + t4 * 4;
+        const uint32_t pbase = sm100::smem_addr(sP) + sb * C::kPBytes + st_row * 128;
+        const int nb = keys / 8;
 #pragma unroll
-        for (int bk = 0; bk < 8; ++bk) {
-          asm volatile("st.shared.b32 [%0], %1;\n" ::"r"(rowa + (((bk ^ ra) & 7) << 4)), "r"(pa[bk]) : "memory");
-          asm volatile("st.shared.b32 [%0], %1;\n" ::"r"(rowb + (((bk ^ rb) & 7) << 4)), "r"(pb[bk]) : "memory");
+        for (int bb = 0; bb < 16; bb += 2) {
+          if (bb < nb) {
+            const int blk = bb + st_blk;
+            const uint32_t addr = pbase + (blk >> 3) * C::kBlock64 + (((blk & 7) ^ (st_row & 7)) << 4);
+            stmatrix_x4(addr, pa[bb], pb[bb], pa[bb + 1], pb[bb + 1]);
+          }
+        }
+      }
+      // Cache rows at or past L in this chunk (the end of the prefix) can
+      // hold anything, NaN included, and P is 0 there: zero their V rows.
+      if (!tree_j && kl < keys) {
+        if (!__all_sync(adt::kFullMask, wait_bar(&bars.v_full[j % NS], (j / NS) & 1, &s_abort, p.err))) break;
+        uint8_t* vt = sStage + (j % NS) * C::kStageBytes + C::kStageTile;
+        const int per_row = C::kBlocks * 8;
+        for (int i = tid; i < (keys - kl) * per_row; i += kSoftmaxWarps * 32) {
+          const int rr = kl + i / per_row, rem = i % per_row;
+          *reinterpret_cast<uint4*>(vt + (rem >> 3) * C::kBlock128 + rr * 128 + (rem & 7) * 16) =
+              make_uint4(0u, 0u, 0u, 0u);
         }
       }
       sm100::fence_proxy_async_smem();
       // Raise O to the new maxima (rare): needs the previous PV product done.
-      if (j > 0 && __any_sync(adt::kFullMask, needa || needb)) {
+      if (j > 0 && __any_sync(adt::kFullMask, alpha_a != 1.f || alpha_b != 1.f)) {
         if (!__all_sync(adt::kFullMask,
-                        wait_bar(&bars.pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, &s_abort, p.err)))
+                        wait_bar(&bars.done[(j - 1) % NS], ((j - 1) / NS) & 1, &s_abort, p.err)))
           break;
         sm100::tc_fence_after();
 #pragma unroll 1
@@ -487,8 +639,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         sm100::tmem_wait_st();
       }
-      mua = nma;
-      mub = nmb;
       sm100::tc_fence_before();
       __syncwarp();
       if (lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.p_full[sb]));
@@ -505,105 +655,105 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   // ------------------------------------------------------------ epilogue
-  // Park this split's partial (O unnormalised, m, l) in shared memory (the
-  // stage ring is idle once O is complete), then merge.
-  constexpr int MS = C::kMergeStride;
-  float* so = reinterpret_cast<float*>(sStage);                         // [64][MS]
-  float2* sml = reinterpret_cast<float2*>(sStage + kMaxNodes * MS * 4);  // [64]
-  float* sw = reinterpret_cast<float*>(sStage + kMaxNodes * MS * 4 + kMaxNodes * 8);  // weights
+  // The softmax threads take their rows of O (unnormalised) into registers.
+  constexpr int kOB = D / 64;
+  uint32_t o[kOB][32];
+  bool have_o = false;
   if (warp < kSoftmaxWarps) {
-    const int g8 = lane >> 2, t4 = lane & 3;
-    const int ra = warp * 16 + g8, rb = ra + 8;
-    // A split without key units (kv_len shorter than max_kv) contributes
-    // nothing: weight 0, zero partial.
-    const bool ok = nu > 0 && !s_abort && __all_sync(adt::kFullMask, wait_bar(&bars.o_full, 0, &s_abort, p.err));
-    if (ok) {
+    const int last = nch - 1;
+    // s_abort can change under the warp: decide once, by a vote.
+    if (__all_sync(adt::kFullMask, nch > 0 && !s_abort))
+      have_o = __all_sync(adt::kFullMask, wait_bar(&bars.done[last % NS], (last / NS) & 1, &s_abort, p.err));
+    if (have_o) {
       sm100::tc_fence_after();
       const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
-#pragma unroll 1
-      for (int c0 = 0; c0 < D; c0 += 64) {
-        uint32_t o[32];
-        tmem_ld_16x256b_x8(tmem + lane_base + kOCol + c0, o);
-        sm100::tmem_wait_ld();
 #pragma unroll
-        for (int bk = 0; bk < 8; ++bk) {
-          const int c = c0 + 8 * bk + 2 * t4;
-          if (ra < n)
-            *reinterpret_cast<float2*>(so + ra * MS + c) = make_float2(__uint_as_float(o[4 * bk]), __uint_as_float(o[4 * bk + 1]));
-          if (rb < n)
-            *reinterpret_cast<float2*>(so + rb * MS + c) =
-                make_float2(__uint_as_float(o[4 * bk + 2]), __uint_as_float(o[4 * bk + 3]));
-        }
-      }
-      if (t4 == 0) {
-        if (ra < n) sml[ra] = make_float2(m_ra, l_ra);
-        if (rb < n) sml[rb] = make_float2(m_rb, l_rb);
-      }
-    } else if (t4 == 0) {
-      for (int half = 0; half < 2; ++half) {
-        const int rr = half ? rb : ra;
-        if (rr < n) {
-          for (int c = 0; c < D; c += 4) *reinterpret_cast<float4*>(so + rr * MS + c) = make_float4(0.f, 0.f, 0.f, 0.f);
-          sml[rr] = make_float2(-INFINITY, 0.f);
-        }
-      }
+      for (int c = 0; c < kOB; ++c) tmem_ld_16x256b_x8(tmem + lane_base + kOCol + c * 64, o[c]);
+      sm100::tmem_wait_ld();
+    } else {
+      // A split without key units (kv_len shorter than max_kv) contributes
+      // nothing: weight 0.
+      m_ra = m_rb = -INFINITY;
+      l_ra = l_rb = 0.f;
     }
   }
   sm100::tc_fence_before();
   __syncthreads();
   if (warp == 0) sm100::tmem_dealloc(tmem, kTmemCols);
 
+  const int g8 = lane >> 2, t4 = lane & 3;
+  const int ra = warp * 16 + g8, rb = ra + 8;
   const int64_t bh = static_cast<int64_t>(b) * p.H + h;
   constexpr int kC4 = D / 4;
   if (p.cluster_merge) {
-    // CTA r of the cluster merges rows r, r + S, ... from every peer's partial.
+    // Split s pushes row r of its partial to split r / rows_per (the row's
+    // owner): slot [s][r % rows_per] of the owner's (m, l) and O arrays, in
+    // the owner's stage ring, which is idle once every split has passed the
+    // first cluster barrier.  After the second, each owner merges its rows.
     cg::cluster_group cl = cg::this_cluster();
+    constexpr int MS = C::kSlotStride;
+    const int rows_per = (n + S - 1) / S;
+    float2* slot_ml = reinterpret_cast<float2*>(sStage);
+    float* slot_o = reinterpret_cast<float*>(sStage + ((S * rows_per * 8 + 15) & ~15));
     cl.sync();
-    const int rank = static_cast<int>(cl.block_rank());
-    const int rows_mine = rank < n ? (n - rank + S - 1) / S : 0;
+    if (warp < kSoftmaxWarps) {
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        const int r = half ? rb : ra;
+        if (r < n) {
+          const int owner = r / rows_per;
+          const int slot = split * rows_per + (r - owner * rows_per);
+          if (t4 == 0) *cl.map_shared_rank(slot_ml + slot, owner) = half ? make_float2(m_rb, l_rb) : make_float2(m_ra, l_ra);
+          if (have_o) {
+            float* dst = cl.map_shared_rank(slot_o, owner) + slot * MS + 2 * t4;
+#pragma unroll
+            for (int c = 0; c < kOB; ++c) {
+#pragma unroll
+              for (int bk = 0; bk < 8; ++bk)
+                *reinterpret_cast<float2*>(dst + c * 64 + 8 * bk) =
+                    make_float2(__uint_as_float(o[c][4 * bk + 2 * half]), __uint_as_float(o[c][4 * bk + 2 * half + 1]));
+            }
+          }
+        }
+      }
+    }
+    cl.sync();
+    const int r_lo = split * rows_per;
+    const int rows_mine = max(0, min(n, r_lo + rows_per) - r_lo);
     if (tid < rows_mine) {
-      const int rr = rank + S * tid;
       float M = -INFINITY;
-      for (int c = 0; c < S; ++c) M = fmaxf(M, cl.map_shared_rank(sml, c)[rr].x);
+      for (int c = 0; c < S; ++c) M = fmaxf(M, slot_ml[c * rows_per + tid].x);
       float lt = 0.f;
       for (int c = 0; c < S; ++c) {
-        const float2 ml = cl.map_shared_rank(sml, c)[rr];
+        const float2 ml = slot_ml[c * rows_per + tid];
         const float w = ml.x == -INFINITY ? 0.f : exp2f(ml.x - M);
-        sw[tid * S + c] = w;
+        s_w[tid * S + c] = w;
         lt += w * ml.y;
       }
       const float inv = 1.f / lt;
-      for (int c = 0; c < S; ++c) sw[tid * S + c] *= inv;
-      if (p.lse) p.lse[static_cast<int64_t>(node0 + rr) * p.H + h] = (M + log2f(lt)) * kLn2;
+      for (int c = 0; c < S; ++c) s_w[tid * S + c] *= inv;
+      if (p.lse) p.lse[static_cast<int64_t>(node0 + r_lo + tid) * p.H + h] = (M + log2f(lt)) * kLn2;
     }
     __syncthreads();
     for (int idx = tid; idx < rows_mine * kC4; idx += kThreads) {
       const int i = idx / kC4, c4 = idx % kC4;
-      const int rr = rank + S * i;
-      // Issue every peer's load before combining (latency, not bandwidth, bound).
-      float4 v[kMaxClusterSplits];
-#pragma unroll
-      for (int c = 0; c < kMaxClusterSplits; ++c) {
-        v[c] = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (c < S && sw[i * S + c] != 0.f)
-          v[c] = *reinterpret_cast<const float4*>(cl.map_shared_rank(so, c) + rr * MS + c4 * 4);
-      }
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-      for (int c = 0; c < kMaxClusterSplits; ++c) {
-        const float w = c < S ? sw[i * S + c] : 0.f;
-        acc.x += w * v[c].x;
-        acc.y += w * v[c].y;
-        acc.z += w * v[c].z;
-        acc.w += w * v[c].w;
+      for (int c = 0; c < S; ++c) {
+        const float w = s_w[i * S + c];
+        if (w != 0.f) {
+          const float4 v = *reinterpret_cast<const float4*>(slot_o + (c * rows_per + i) * MS + c4 * 4);
+          acc.x += w * v.x;
+          acc.y += w * v.y;
+          acc.z += w * v.z;
+          acc.w += w * v.w;
+        }
       }
-      __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + rr) * p.H + h) * D + c4 * 4;
+      __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + r_lo + i) * p.H + h) * D + c4 * 4;
       uint2 pk;
       pk.x = pack_bf16x2(acc.x, acc.y);
       pk.y = pack_bf16x2(acc.z, acc.w);
       *reinterpret_cast<uint2*>(dst) = pk;
     }
-    cl.sync();  // peers may still be reading this CTA's partial
     return;
   }
 
@@ -611,11 +761,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   // and the CTA that finishes a (tree, head) last merges them.
   float* po = p.part_o + (bh * S + split) * kMaxNodes * D;
   float2* pml = p.part_ml + (bh * S + split) * kMaxNodes;
-  for (int idx = tid; idx < n * kC4; idx += kThreads) {
-    const int rr = idx / kC4, c4 = idx % kC4;
-    *reinterpret_cast<float4*>(po + rr * D + c4 * 4) = *reinterpret_cast<const float4*>(so + rr * MS + c4 * 4);
+  if (warp < kSoftmaxWarps) {
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+      const int r = half ? rb : ra;
+      if (r < n) {
+        if (t4 == 0) pml[r] = half ? make_float2(m_rb, l_rb) : make_float2(m_ra, l_ra);
+#pragma unroll
+        for (int c = 0; c < kOB; ++c) {
+#pragma unroll
+          for (int bk = 0; bk < 8; ++bk) {
+            const float2 v = have_o ? make_float2(__uint_as_float(o[c][4 * bk + 2 * half]),
+                                                  __uint_as_float(o[c][4 * bk + 2 * half + 1]))
+                                    : make_float2(0.f, 0.f);
+            *reinterpret_cast<float2*>(po + r * D + c * 64 + 8 * bk + 2 * t4) = v;
+          }
+        }
+      }
+    }
   }
-  if (tid < n) pml[tid] = sml[tid];
   __threadfence();
   __syncthreads();
   if (tid == 0) s_last = atomicAdd(p.tickets + bh, 1u) == static_cast<unsigned>(S - 1);
@@ -624,8 +788,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __threadfence();
   const float* po_bh = p.part_o + bh * S * kMaxNodes * D;
   const float2* pml_bh = p.part_ml + bh * S * kMaxNodes;
-  float* wsm = reinterpret_cast<float*>(sStage);  // [64][S]; the parked partial is in global now
-  __syncthreads();
+  float* wsm = reinterpret_cast<float*>(sStage);  // [64][S]
   if (tid < n) {
     float M = -INFINITY;
     for (int sp = 0; sp < S; ++sp) M = fmaxf(M, __ldcg(&pml_bh[sp * kMaxNodes + tid]).x);
