@@ -75,15 +75,16 @@ struct Cfg {
   static constexpr int kStageBytes = 2 * kStageTile;     // K tile, then V tile
   static constexpr int kPBytes = 2 * kBlock64;           // 64 query rows x 128 keys
   static constexpr int kStages = D == 128 ? 2 : 4;
+  static constexpr int kRowStride = D + 8;               // fp32 per merged row: D values, m, l, pad
   static constexpr int kQOff = 0;
   static constexpr int kPOff = kTreeTile;                // Q is 64 rows x D, like a tree tile
-  static constexpr int kTreeOff = kPOff + 2 * kPBytes;   // tree unit: K tile, then V tile
-  static constexpr int kStageOff = kTreeOff + 2 * kTreeTile;
-  static constexpr int kDynSmem = kStageOff + kStages * kStageBytes + 1024;  // + alignment slack
+  static constexpr int kStageOff = kPOff + 2 * kPBytes;  // the tree unit's K/V go to slot 0
+  static constexpr int kSlotOff = kStageOff + kStages * kStageBytes;  // incoming rows of the merge
+  static constexpr int kSlotBytes = (kMaxNodes + kMaxClusterSplits) * kRowStride * 4;
+  static constexpr int kDynSmem = kSlotOff + kSlotBytes + 1024;  // + alignment slack
   static constexpr uint32_t kIdescS128 = sm100::idesc_bf16_f32(64, 128, 0, 0);
   static constexpr uint32_t kIdescS64 = sm100::idesc_bf16_f32(64, 64, 0, 0);
   static constexpr uint32_t kIdescO = sm100::idesc_bf16_f32(64, D, 0, 1);
-  static constexpr int kSlotStride = D + 8;  // fp32 per pushed row: conflict-free float2 stores
   static_assert(kStages <= kMaxStages, "stage ring");
 };
 
@@ -105,11 +106,11 @@ struct TcParams {
   unsigned* err;
 };
 
-// Byte offset of 16-byte chunk `ch` (0 .. D/8-1) of row `row` in a 64-row
-// tile of 128-byte column blocks with the 128-byte swizzle (the layout TMA
-// writes).
-__device__ __forceinline__ uint32_t sw128_off(int row, int ch) {
-  return static_cast<uint32_t>((ch >> 3) * (kUnit * 128) + row * 128 + (((ch & 7) ^ (row & 7)) << 4));
+// Byte offset of 16-byte chunk `ch` (0 .. D/8-1) of row `row` in a tile of
+// 128-byte column blocks of `block_rows` rows with the 128-byte swizzle (the
+// layout TMA writes).
+__device__ __forceinline__ uint32_t sw128_off(int row, int ch, int block_rows) {
+  return static_cast<uint32_t>((ch >> 3) * block_rows * 128 + row * 128 + (((ch & 7) ^ (row & 7)) << 4));
 }
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, int src_bytes) {
@@ -247,6 +248,7 @@ struct Barriers {
   uint64_t s_free[2];
   uint64_t p_full[2];
   uint64_t drain[2];               // abort path: every MMA a thread issued finished
+  uint64_t recv;                   // cluster merge: every split's rows for this owner landed
 };
 
 // Bounded wait that also gives up when another role has aborted.
@@ -267,12 +269,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                         const TcParams p) {
   using C = Cfg<D>;
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  // 1024-byte aligned for the 128-byte swizzle; pointer arithmetic on the
+  // shared array keeps accesses in the shared address space.
+  uint8_t* smem = smem_raw + ((1024u - (sm100::smem_addr(smem_raw) & 1023u)) & 1023u);
   __shared__ Barriers bars;
   __shared__ uint64_t anc[kMaxNodes];
   __shared__ int s_par[kMaxNodes];
-  __shared__ float s_w[kMaxNodes + kMaxClusterSplits];
   __shared__ uint32_t tmem_slot;
   __shared__ int s_bad;
   __shared__ int s_last;
@@ -297,28 +300,29 @@ __global__ void __launch_bounds__(kThreads, 1)
     return;
   }
 
-  const int U = (L + kUnit - 1) / kUnit + 1;  // prefix units + the tree unit
+  // The keys are cut into chunks: ceil(P / 2) prefix chunks of two 64-key
+  // units (P = ceil(L / 64); the last holds one unit when P is odd) and the
+  // tree unit.  Split s takes chunks [s T / S, (s + 1) T / S) of the T; the
+  // split whose share ends with the tree unit processes it first.
+  const int P = (L + kUnit - 1) / kUnit;
+  const int T = (P + 1) / 2 + 1;
   const int S = p.splits;
-  const int u_begin = static_cast<int>(static_cast<int64_t>(split) * U / S);
-  const int u_end = static_cast<int>(static_cast<int64_t>(split + 1) * U / S);
-  const int nu = u_end - u_begin;
-  // Chunk 0 is the tree unit for the CTA whose share ends with it; prefix
-  // units follow two per chunk (the last chunk may hold one).
-  const int has_tree = (u_end == U && nu > 0) ? 1 : 0;
-  const int np = nu - has_tree;  // prefix units of this CTA
-  const int nch = has_tree + (np + 1) / 2;
+  const int c_begin = static_cast<int>(static_cast<int64_t>(split) * T / S);
+  const int c_end = static_cast<int>(static_cast<int64_t>(split + 1) * T / S);
+  const int nch = c_end - c_begin;
+  const int has_tree = (c_end == T && nch > 0) ? 1 : 0;
   const int NS = C::kStages;
   auto chunk_keys = [&](int j) -> int {
     if (has_tree && j == 0) return kUnit;
-    const int pc = j - has_tree;
-    return (np - 2 * pc >= 2 ? 2 : 1) * kUnit;
+    const int pc = c_begin + j - has_tree;
+    return (2 * pc + 1 < P ? 2 : 1) * kUnit;
   };
-  auto chunk_key0 = [&](int j) -> int { return (u_begin + 2 * (j - has_tree)) * kUnit; };
+  auto chunk_key0 = [&](int j) -> int { return (c_begin + j - has_tree) * kChunk; };
 
   uint8_t* sQ = smem + C::kQOff;
   uint8_t* sP = smem + C::kPOff;
   uint8_t* sStage = smem + C::kStageOff;
-  uint8_t* sTree = smem + C::kTreeOff;
+  float* slots = reinterpret_cast<float*>(smem + C::kSlotOff);  // merge: [S][rows_per][kRowStride]
 
   if (tid == 0) {
     s_bad = 0;
@@ -337,6 +341,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     sm100::mbar_init(sm100::smem_addr(&bars.drain[0]), 1);
     sm100::mbar_init(sm100::smem_addr(&bars.drain[1]), 1);
+    sm100::mbar_init(sm100::smem_addr(&bars.recv), 1);
     sm100::fence_mbar_init();
   }
   if (warp == 0) {
@@ -345,17 +350,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (warp < kSoftmaxWarps) {
     // Q tile: rows node0 .. node0+63 (rows past the tree zero-filled); the
-    // tree unit's K/V for kv head g likewise; the parent pointers.
+    // tree unit's K/V for kv head g likewise, into stage slot 0 (the tree is
+    // chunk 0); the parent pointers.
     for (int i = tid; i < kUnit * (D / 8); i += kSoftmaxWarps * 32) {
       const int r = i / (D / 8), ch = i % (D / 8);
       const bool valid = r < n;
       const int row = node0 + (valid ? r : 0);
-      cp_async16(sm100::smem_addr(sQ) + sw128_off(r, ch), p.q + (static_cast<int64_t>(row) * p.H + h) * D + ch * 8,
-                 valid ? 16 : 0);
+      cp_async16(sm100::smem_addr(sQ) + sw128_off(r, ch, kUnit),
+                 p.q + (static_cast<int64_t>(row) * p.H + h) * D + ch * 8, valid ? 16 : 0);
       if (has_tree) {
         const int64_t off = (static_cast<int64_t>(row) * p.Hkv + g) * D + ch * 8;
-        cp_async16(sm100::smem_addr(sTree) + sw128_off(r, ch), p.kt + off, valid ? 16 : 0);
-        cp_async16(sm100::smem_addr(sTree + C::kTreeTile) + sw128_off(r, ch), p.vt + off, valid ? 16 : 0);
+        cp_async16(sm100::smem_addr(sStage) + sw128_off(r, ch, kChunk), p.kt + off, valid ? 16 : 0);
+        cp_async16(sm100::smem_addr(sStage + C::kStageTile) + sw128_off(r, ch, kChunk), p.vt + off, valid ? 16 : 0);
       }
     }
     if (tid < n) cp_async4(sm100::smem_addr(&s_par[tid]), p.parents + node0 + tid);
@@ -364,6 +370,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   sm100::tc_fence_after();
   const uint32_t tmem = tmem_slot;
+  // The mbarriers are initialised: tell the cluster (the merge's bulk copies
+  // complete on a peer's barrier; every thread waits on this before one).
+  sm100::cluster_arrive_relaxed();
 
   // Stage loads: chunk j goes to slot j % NS, K tile by warp 4 and V tile by
   // warp 6.  The tree chunk loads nothing (its K/V came with Q) but still
@@ -469,14 +478,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             (j >= 2 && !wait_bar(&bars.s_free[sb], ((j >> 1) - 1) & 1, &s_abort, p.err)))
           break;
         sm100::tc_fence_after();
-        const bool tree_j = has_tree && j == 0;
-        const uint32_t k_addr = tree_j ? sm100::smem_addr(sTree) : sm100::smem_addr(sStage + st * C::kStageBytes);
-        const uint32_t k_blk = tree_j ? C::kBlock64 : C::kBlock128;
+        const uint32_t k_addr = sm100::smem_addr(sStage + st * C::kStageBytes);
         const uint32_t idesc = chunk_keys(j) == kChunk ? C::kIdescS128 : C::kIdescS64;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint64_t da = sm100::smem_desc_sw128(q_addr + (kk >> 2) * C::kBlock64 + (kk & 3) * 32, 16, 1024);
-          const uint64_t db = sm100::smem_desc_sw128(k_addr + (kk >> 2) * k_blk + (kk & 3) * 32, 16, 1024);
+          const uint64_t db = sm100::smem_desc_sw128(k_addr + (kk >> 2) * C::kBlock128 + (kk & 3) * 32, 16, 1024);
           sm100::mma_bf16_ss(tmem + sb * kSCols, da, db, idesc, kk > 0 ? 1u : 0u);
         }
         sm100::mma_commit(sm100::smem_addr(&bars.s_full[sb]));
@@ -500,15 +507,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             !wait_bar(&bars.v_full[i % NS], (i / NS) & 1, &s_abort, p.err))
           break;
         sm100::tc_fence_after();
-        const bool tree_i = has_tree && i == 0;
-        const uint32_t v_addr = tree_i ? sm100::smem_addr(sTree + C::kTreeTile)
-                                       : sm100::smem_addr(sStage + (i % NS) * C::kStageBytes + C::kStageTile);
-        const uint32_t v_lbo = tree_i ? C::kBlock64 : C::kBlock128;  // stride of V's d blocks
+        const uint32_t v_addr = sm100::smem_addr(sStage + (i % NS) * C::kStageBytes + C::kStageTile);
         const uint32_t pb = p_addr + (i & 1) * C::kPBytes;
         const int ksteps = chunk_keys(i) / 16;
         for (int kk = 0; kk < ksteps; ++kk) {
           const uint64_t da = sm100::smem_desc_sw128(pb + (kk >> 2) * C::kBlock64 + (kk & 3) * 32, 16, 1024);
-          const uint64_t db = sm100::smem_desc_sw128(v_addr + kk * 2048, v_lbo, 1024);
+          const uint64_t db = sm100::smem_desc_sw128(v_addr + kk * 2048, C::kBlock128, 1024);  // LBO: d blocks
           sm100::mma_bf16_ss(tmem + kOCol, da, db, C::kIdescO, (i > 0 || kk > 0) ? 1u : 0u);
         }
         sm100::mma_commit(sm100::smem_addr(&bars.done[i % NS]));
@@ -678,82 +682,108 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   sm100::tc_fence_before();
-  __syncthreads();
-  if (warp == 0) sm100::tmem_dealloc(tmem, kTmemCols);
 
   const int g8 = lane >> 2, t4 = lane & 3;
   const int ra = warp * 16 + g8, rb = ra + 8;
   const int64_t bh = static_cast<int64_t>(b) * p.H + h;
   constexpr int kC4 = D / 4;
   if (p.cluster_merge) {
-    // Split s pushes row r of its partial to split r / rows_per (the row's
-    // owner): slot [s][r % rows_per] of the owner's (m, l) and O arrays, in
-    // the owner's stage ring, which is idle once every split has passed the
-    // first cluster barrier.  After the second, each owner merges its rows.
-    cg::cluster_group cl = cg::this_cluster();
-    constexpr int MS = C::kSlotStride;
+    // Row r of the (tree, head) is merged by split r / rows_per, its owner.
+    // Each split writes its partial rows (O unnormalised, then m and l) into
+    // its own stage ring, idle now, in row order; one thread sends every
+    // owner its rows with bulk shared-to-shared copies into the owner's slot
+    // region, completing on the owner's mbarrier; each owner merges locally.
+    constexpr int RS = C::kRowStride;
     const int rows_per = (n + S - 1) / S;
-    float2* slot_ml = reinterpret_cast<float2*>(sStage);
-    float* slot_o = reinterpret_cast<float*>(sStage + ((S * rows_per * 8 + 15) & ~15));
-    cl.sync();
+    const int r_lo = split * rows_per;
+    const int rows_mine = max(0, min(n, r_lo + rows_per) - r_lo);
+    float* rows_out = reinterpret_cast<float*>(sStage);
+    if (tid == 0)
+      sm100::mbar_arrive_expect_tx(sm100::smem_addr(&bars.recv), static_cast<uint32_t>(S * rows_mine * RS * 4));
     if (warp < kSoftmaxWarps) {
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
         const int r = half ? rb : ra;
         if (r < n) {
-          const int owner = r / rows_per;
-          const int slot = split * rows_per + (r - owner * rows_per);
-          if (t4 == 0) *cl.map_shared_rank(slot_ml + slot, owner) = half ? make_float2(m_rb, l_rb) : make_float2(m_ra, l_ra);
-          if (have_o) {
-            float* dst = cl.map_shared_rank(slot_o, owner) + slot * MS + 2 * t4;
+          float* dst = rows_out + r * RS;
+          if (t4 == 0) *reinterpret_cast<float2*>(dst + D) = half ? make_float2(m_rb, l_rb) : make_float2(m_ra, l_ra);
 #pragma unroll
-            for (int c = 0; c < kOB; ++c) {
+          for (int c = 0; c < kOB; ++c) {
 #pragma unroll
-              for (int bk = 0; bk < 8; ++bk)
-                *reinterpret_cast<float2*>(dst + c * 64 + 8 * bk) =
-                    make_float2(__uint_as_float(o[c][4 * bk + 2 * half]), __uint_as_float(o[c][4 * bk + 2 * half + 1]));
-            }
+            for (int bk = 0; bk < 8; ++bk)
+              *reinterpret_cast<float2*>(dst + c * 64 + 8 * bk + 2 * t4) =
+                  have_o ? make_float2(__uint_as_float(o[c][4 * bk + 2 * half]),
+                                       __uint_as_float(o[c][4 * bk + 2 * half + 1]))
+                         : make_float2(0.f, 0.f);
           }
         }
       }
+      sm100::fence_proxy_async_smem();
+      softmax_warps_sync();
     }
-    cl.sync();
-    const int r_lo = split * rows_per;
-    const int rows_mine = max(0, min(n, r_lo + rows_per) - r_lo);
-    if (tid < rows_mine) {
-      float M = -INFINITY;
-      for (int c = 0; c < S; ++c) M = fmaxf(M, slot_ml[c * rows_per + tid].x);
-      float lt = 0.f;
+    // Pairs with the arrive after the prologue: every peer's receive barrier
+    // is initialised.
+    sm100::cluster_wait_acquire();
+    if (tid == 0) {
       for (int c = 0; c < S; ++c) {
-        const float2 ml = slot_ml[c * rows_per + tid];
-        const float w = ml.x == -INFINITY ? 0.f : exp2f(ml.x - M);
-        s_w[tid * S + c] = w;
-        lt += w * ml.y;
+        const int rc = max(0, min(n, (c + 1) * rows_per) - c * rows_per);
+        if (rc > 0)
+          sm100::bulk_copy_to_cluster(sm100::mapa_shared(sm100::smem_addr(slots + split * rows_per * RS), c),
+                                      sm100::smem_addr(rows_out + c * rows_per * RS),
+                                      static_cast<uint32_t>(rc * RS * 4),
+                                      sm100::mapa_shared(sm100::smem_addr(&bars.recv), c));
       }
-      const float inv = 1.f / lt;
-      for (int c = 0; c < S; ++c) s_w[tid * S + c] *= inv;
-      if (p.lse) p.lse[static_cast<int64_t>(node0 + r_lo + tid) * p.H + h] = (M + log2f(lt)) * kLn2;
     }
-    __syncthreads();
+    // Not abandoned on an abort elsewhere: copies into this CTA's shared
+    // memory must have landed before it exits.
+    if (!sm100::mbar_wait_bounded(sm100::smem_addr(&bars.recv), 0, kWaitLimit) && tid == 0)
+      adt::raise_error(p.err, ADT_DEVERR_TIMEOUT);
+    // This owner has its rows, so the copies it was sent are complete.
+    sm100::cluster_arrive_relaxed();
+    // Thread (row i, column group c4) combines the S partials of that row:
+    // weights 2^(m_c - M) l_c / sum, every split's values loaded up front.
+    // A split without keys sent zeros with m = -inf (weight 0).
     for (int idx = tid; idx < rows_mine * kC4; idx += kThreads) {
       const int i = idx / kC4, c4 = idx % kC4;
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int c = 0; c < S; ++c) {
-        const float w = s_w[i * S + c];
-        if (w != 0.f) {
-          const float4 v = *reinterpret_cast<const float4*>(slot_o + (c * rows_per + i) * MS + c4 * 4);
-          acc.x += w * v.x;
-          acc.y += w * v.y;
-          acc.z += w * v.z;
-          acc.w += w * v.w;
+      float2 ml[kMaxClusterSplits];
+      float4 v[kMaxClusterSplits];
+#pragma unroll
+      for (int c = 0; c < kMaxClusterSplits; ++c) {
+        if (c < S) {
+          const float* row = slots + (c * rows_per + i) * RS;
+          ml[c] = *reinterpret_cast<const float2*>(row + D);
+          v[c] = *reinterpret_cast<const float4*>(row + c4 * 4);
+        } else {
+          ml[c] = make_float2(-INFINITY, 0.f);
+          v[c] = make_float4(0.f, 0.f, 0.f, 0.f);
         }
       }
+      float M = ml[0].x;
+#pragma unroll
+      for (int c = 1; c < kMaxClusterSplits; ++c) M = fmaxf(M, ml[c].x);
+      float lt = 0.f;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int c = 0; c < kMaxClusterSplits; ++c) {
+        const float w = ml[c].x == -INFINITY ? 0.f : ex2_approx(ml[c].x - M);
+        lt += w * ml[c].y;
+        acc.x += w * v[c].x;
+        acc.y += w * v[c].y;
+        acc.z += w * v[c].z;
+        acc.w += w * v[c].w;
+      }
+      const float inv = 1.f / lt;
       __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + r_lo + i) * p.H + h) * D + c4 * 4;
       uint2 pk;
-      pk.x = pack_bf16x2(acc.x, acc.y);
-      pk.y = pack_bf16x2(acc.z, acc.w);
+      pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+      pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
       *reinterpret_cast<uint2*>(dst) = pk;
+      if (c4 == 0 && p.lse) p.lse[static_cast<int64_t>(node0 + r_lo + i) * p.H + h] = (M + log2f(lt)) * kLn2;
     }
+    // Every owner has its rows: this CTA's outgoing copies are complete.
+    sm100::cluster_wait_acquire();
+    sm100::tc_fence_after();
+    if (warp == 0) sm100::tmem_dealloc(tmem, kTmemCols);
     return;
   }
 
@@ -781,7 +811,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   __threadfence();
+  sm100::cluster_wait_acquire();  // pairs with the prologue's arrive (a cluster of one CTA here)
   __syncthreads();
+  sm100::tc_fence_after();
+  if (warp == 0) sm100::tmem_dealloc(tmem, kTmemCols);
   if (tid == 0) s_last = atomicAdd(p.tickets + bh, 1u) == static_cast<unsigned>(S - 1);
   __syncthreads();
   if (!s_last) return;
@@ -842,7 +875,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ---------------------------------------------------------------- host side
 
-// Splits per (tree, head): about one CTA per SM, at most one split per unit
+// Splits per (tree, head): about one CTA per SM, at most one split per chunk
 // of keys.  Up to kMaxClusterSplits splits form a cluster; the count is
 // lowered until all B*H clusters are co-resident (GPC sizes decide how many
 // clusters of a given size fit at once).  Many splits (small B*H, long
@@ -850,7 +883,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 int max_active_clusters(int D, int cluster, int dev);
 
 int choose_splits(int sm_count, int B, int H, int D, int max_kv, int dev) {
-  const int units = (max_kv + kUnit - 1) / kUnit + 1;
+  const int units = ((max_kv + kUnit - 1) / kUnit + 1) / 2 + 1;  // chunks, the tree unit included
   const int bh = B * H;
   int s = sm_count / bh;
   if (s < 1) s = 1;
