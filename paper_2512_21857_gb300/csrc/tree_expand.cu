@@ -2,28 +2,44 @@
 // (Sec. 3.1, last paragraph; Fig. 5; node score Eq. 4 in the log domain), and
 // adt_tree_rerank: the final top-N tree (Eq. 4 and the sentence after it).
 //
-// Expand is one launch over (vocab chunk, frontier row).  Each CTA stages a
-// 4096-logit chunk in shared memory, computes the chunk's max and sum of
-// exponentials and its exact top-k by radix selection on 64-bit keys
-// (value order, then lower index), and writes them to the workspace.  The
-// last CTA of a row (atomic ticket) merges the chunk results into the row's
-// top-k and log-sum-exp and writes the children; the last row to finish
-// selects the next frontier across all rows the same way.
+// Expand is one launch of F thread-block clusters, one per frontier row; the
+// C <= 8 CTAs of a cluster split the row's vocabulary.  Each warp streams its
+// share of the logits (x / T in fp32, round-to-nearest division) keeping a
+// running maximum and sum of exponentials and each lane's two largest
+// selection keys (value order, then lower index).  The k-th largest of the
+// warp's 64 lane keys bounds the warp's top k from below; a second pass
+// gathers the keys at or above it and ranks them.  Sorted lists then merge by
+// rank (binary search in the other lists): the warps' into the CTA's, the
+// CTAs' into the cluster's first CTA through distributed shared memory, which
+// writes the row's children (log-probability against the row's log-sum-exp
+// in fp64).  The first CTA of the last row to finish (atomic ticket) selects
+// the next frontier across all rows the same way.
+#include <cooperative_groups.h>
+
 #include "adt_common.cuh"
+#include "sm100.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kChunk = 4096;
+constexpr int kWarps = kThreads / 32;
 constexpr int kMaxK = 64;
 constexpr int kMaxKeep = 1024;
+constexpr int kMaxCluster = 8;
+constexpr int kValuesPerCta = 2048;     // a CTA per this many logits, up to kMaxCluster per row
+constexpr int kTile = 16384;            // logits staged in shared memory at a time
+constexpr uint32_t kWaitLimit = 1u << 22;
+constexpr int kCandCap = 1024;          // a CTA's candidate buffer (also the cross-row keys)
+constexpr float kLog2e = 1.44269504088896340736f;
 
 struct ExpandParams {
   const float* logits;
   int64_t ld;
   const float* fscore;
   const int32_t* fid;
-  int F, V, k, k_keep, S;
+  int F, V, k, k_keep;
   float T;
   int use_T;
   int32_t id_base;
@@ -34,13 +50,40 @@ struct ExpandParams {
   int32_t* keep;
   float* nscore;
   int32_t* nid;
-  uint64_t* part_keys;  // [F][S][k]
-  float* part_max;      // [F][S]
-  double* part_sum;     // [F][S]
-  uint64_t* cross_keys; // [F*k]
-  unsigned* row_tickets;  // [F]
+  uint64_t* cross_keys;   // [F*k]
   unsigned* all_ticket;   // [1]
+  unsigned* err;
 };
+
+// Entries greater than key in a descending list of n keys.
+__device__ __forceinline__ int count_greater(const uint64_t* list, int n, uint64_t key) {
+  int lo = 0, hi = n;
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (list[mid] > key)
+      lo = mid + 1;
+    else
+      hi = mid;
+  }
+  return lo;
+}
+
+// Top k of nl descending lists (list l at lists + l * stride, its first len
+// entries; 0 pads) into out[0..k), which the caller zeroed.  Keys are
+// distinct, so an entry's rank is its index plus the entries greater than it
+// in the other lists.
+__device__ void merge_topk(const uint64_t* lists, int nl, int stride, int len, int k, uint64_t* out) {
+  const int lk = min(len, k);
+  for (int c = threadIdx.x; c < nl * lk; c += kThreads) {
+    const int l = c / lk, j = c % lk;
+    const uint64_t key = lists[l * stride + j];
+    if (key == 0ull) continue;
+    int rank = j;
+    for (int l2 = 0; l2 < nl && rank < k; ++l2)
+      if (l2 != l) rank += count_greater(lists + l2 * stride, lk, key);
+    if (rank < k) out[rank] = key;
+  }
+}
 
 // Collects the keys >= thr (exactly `count` of them) into sel[] and sorts
 // them in descending order (padding with 0 up to a power of two).
@@ -62,93 +105,287 @@ __device__ void collect_sorted(KeyAt key_at, int n, uint64_t thr, int count, uin
   adt::block_bitonic_sort_desc<kThreads>(sel, P);
 }
 
+// The k (<= 64) largest keys a warp is offered, kept sorted by insertion:
+// lane i holds entries i (a) and i + 32 (b); 0 marks an empty entry.  Used
+// only when a warp's candidate buffer overflows (inputs with very many keys
+// at or above the warp's bound).
+struct WarpTopK {
+  uint64_t a = 0, b = 0;
+  __device__ __forceinline__ uint64_t threshold(int k) const {
+    const int i = k - 1;
+    return __shfl_sync(adt::kFullMask, i < 32 ? a : b, i & 31);
+  }
+  __device__ __forceinline__ void insert(uint64_t key, int k, int lane) {
+    const int pos = __popc(__ballot_sync(adt::kFullMask, a > key)) + __popc(__ballot_sync(adt::kFullMask, b > key));
+    if (pos >= k) return;
+    const uint64_t up_a = __shfl_up_sync(adt::kFullMask, a, 1);
+    const uint64_t up_b = __shfl_up_sync(adt::kFullMask, b, 1);
+    const uint64_t a31 = __shfl_sync(adt::kFullMask, a, 31);
+    const int ia = lane, ib = lane + 32;
+    const uint64_t na = ia < pos ? a : (ia == pos ? key : up_a);
+    const uint64_t nb = ib < pos ? b : (ib == pos ? key : (lane == 0 ? a31 : up_b));
+    a = ia < k ? na : 0ull;
+    b = ib < k ? nb : 0ull;
+  }
+  __device__ __forceinline__ void offer(uint64_t key, int k, int lane, uint64_t& thr) {
+    unsigned m = __ballot_sync(adt::kFullMask, key > thr);
+    while (m) {
+      const int src = __ffs(m) - 1;
+      insert(__shfl_sync(adt::kFullMask, key, src), k, lane);
+      thr = threshold(k);
+      m &= m - 1;
+      m &= __ballot_sync(adt::kFullMask, key > thr);
+    }
+  }
+};
+
+// Stages logits [t0, t1) of a row (t0 a multiple of 4; rows start 16-byte
+// aligned and ld is a multiple of 4) in shared memory with one bulk copy,
+// waiting with a bound.  Then divides by the temperature in place.  Block-wide.
+__device__ bool stage_tile(float* vals, const float* row, int t0, int t1, const ExpandParams& p, uint64_t* bar,
+                           uint32_t& phase) {
+  const int n = t1 - t0;
+  if (threadIdx.x == 0 && n > 0) {
+    const uint32_t bytes = static_cast<uint32_t>((n + 3) / 4 * 16);
+    sm100::mbar_arrive_expect_tx(sm100::smem_addr(bar), bytes);
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(
+            sm100::smem_addr(vals)),
+        "l"(row + t0), "r"(bytes), "r"(sm100::smem_addr(bar))
+        : "memory");
+  }
+  bool ok = true;
+  if (n > 0) {
+    ok = sm100::mbar_wait_bounded(sm100::smem_addr(bar), phase, kWaitLimit);
+    phase ^= 1u;
+  }
+  if (p.use_T) {
+    for (int i = threadIdx.x; i < n; i += kThreads) vals[i] = __fdiv_rn(vals[i], p.T);
+  }
+  __syncthreads();
+  return ok;
+}
+
+// out[rank] = key for the k largest of the n distinct nonzero keys in
+// keys[0..n) (0 entries skipped); out[] zeroed by the caller.  Block-wide:
+// every key counts the keys above it (broadcast reads, no dependent loads).
+__device__ void rank_select(const uint64_t* keys, int n, int k, uint64_t* out) {
+  for (int i = threadIdx.x; i < n; i += kThreads) {
+    const uint64_t key = keys[i];
+    if (key == 0ull) continue;
+    int rk = 0;
+#pragma unroll 8
+    for (int j = 0; j < n; ++j) rk += keys[j] > key;
+    if (rk < k) out[rk] = key;
+  }
+}
+
+// 2^x with the hardware approximation (flush-to-zero); 2^-inf = 0.
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;\n" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// The k-th largest (k <= 32) of the warp's 32 values, by a bitonic sort
+// across the lanes (descending).
+__device__ __forceinline__ float warp_kth_largest(float v, int k, int lane) {
+#pragma unroll
+  for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      const float o = __shfl_xor_sync(adt::kFullMask, v, stride);
+      const bool keep_max = ((lane & stride) == 0) == ((lane & size) == 0);
+      v = keep_max ? fmaxf(v, o) : fminf(v, o);
+    }
+  }
+  return __shfl_sync(adt::kFullMask, v, k - 1);
+}
+
 __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) {
-  __shared__ float vals[kChunk];
-  __shared__ uint64_t sel[kMaxKeep];
-  __shared__ adt::RadixScratch rs;
-  __shared__ double dred[32];
-  __shared__ float fred[32];
+  extern __shared__ __align__(16) float vals[];    // [min(per, kTile)] staged logits
+  __shared__ uint64_t cand[kCandCap];              // keys at or above the CTA's bound
+  __shared__ uint64_t wl[kWarps][kMaxK];           // overflow path: each warp's top k
+  __shared__ float s_bw[kWarps], s_mw[kWarps], s_sw[kWarps];
   __shared__ unsigned s_cnt;
+  __shared__ uint64_t ctl[kMaxK];                  // this CTA's top k
+  __shared__ uint64_t cl_keys[kMaxCluster * kMaxK];  // first CTA of the cluster: every CTA's k keys
+  __shared__ float2 cl_ms[kMaxCluster];
+  __shared__ uint64_t rowl[kMaxK];
+  __shared__ adt::RadixScratch rs;
+  __shared__ __align__(8) uint64_t s_bar;
   __shared__ int s_last;
   __shared__ double s_lse;
+  uint64_t* cross_s = cand;  // cross-row keys (reuses the candidate buffer)
+  uint64_t* sel = cand;      // radix path [kMaxKeep]
 
-  const int s = blockIdx.x, r = blockIdx.y, tid = threadIdx.x;
-  const int t0 = s * kChunk;
-  const int len = min(kChunk, p.V - t0);
+  cg::cluster_group cl = cg::this_cluster();
+  const int rank = blockIdx.x, C = gridDim.x, r = blockIdx.y;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int K = p.k;
+  // This CTA's share of the row: [c0, c1), c0 a multiple of 4.
+  const int per = (((p.V + C - 1) / C) + 3) & ~3;
+  const int c0 = min(p.V, rank * per), c1 = min(p.V, c0 + per);
+  const int ntiles = (c1 - c0 + kTile - 1) / kTile;
   const float* row = p.logits + static_cast<int64_t>(r) * p.ld;
 
-  // Stage the chunk (x / T in fp32, round-to-nearest division).
-  for (int i = tid * 4; i < len; i += kThreads * 4) {
-    float x[4];
-    if (i + 3 < len) {
-      const float4 v = __ldg(reinterpret_cast<const float4*>(row + t0 + i));
-      x[0] = v.x; x[1] = v.y; x[2] = v.z; x[3] = v.w;
-    } else {
-      for (int e = 0; e < 4; ++e) x[e] = (i + e < len) ? __ldg(row + t0 + i + e) : 0.f;
-    }
-    for (int e = 0; e < 4 && i + e < len; ++e) vals[i + e] = p.use_T ? __fdiv_rn(x[e], p.T) : x[e];
-  }
-  __syncthreads();
-
-  float m = -INFINITY;
-  for (int i = tid; i < len; i += kThreads) m = fmaxf(m, vals[i]);
-  m = adt::block_max<kThreads>(m, fred);
-  float acc = 0.f;
-  for (int i = tid; i < len; i += kThreads) acc += expf(vals[i] - m);
-  const double tot = adt::block_sum<kThreads, double>(static_cast<double>(acc), dred);
-
-  const int kk = min(p.k, len);
-  auto chunk_key = [&](int i) { return adt::select_key(vals[i], static_cast<uint32_t>(t0 + i)); };
-  const uint64_t thr = adt::block_topk_threshold<kThreads>(chunk_key, len, kk, &rs);
-  collect_sorted(chunk_key, len, thr, kk, sel, &s_cnt);
-
-  const int64_t rs_idx = static_cast<int64_t>(r) * p.S + s;
-  for (int j = tid; j < p.k; j += kThreads) p.part_keys[rs_idx * p.k + j] = j < kk ? sel[j] : 0ull;
+  for (int i = tid; i < kMaxK; i += kThreads) ctl[i] = 0ull;
   if (tid == 0) {
-    p.part_max[rs_idx] = m;
-    p.part_sum[rs_idx] = tot;
+    s_cnt = 0u;
+    sm100::mbar_init(sm100::smem_addr(&s_bar), 1);
+    sm100::fence_mbar_init();
   }
-  __threadfence();
   __syncthreads();
-  if (tid == 0) s_last = atomicAdd(p.row_tickets + r, 1u) == static_cast<unsigned>(p.S - 1);
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
+  uint32_t phase = 0;
+  bool ok = true;
 
-  // ---- last CTA of row r: merge chunk results.
-  const uint64_t* rk = p.part_keys + static_cast<int64_t>(r) * p.S * p.k;
-  auto row_key = [&](int i) { return __ldcg(rk + i); };
-  const uint64_t thr2 = adt::block_topk_threshold<kThreads>(row_key, p.S * p.k, p.k, &rs);
-  collect_sorted(row_key, p.S * p.k, thr2, p.k, sel, &s_cnt);
-  if (tid < 32) {
-    double M = -INFINITY;
-    for (int c = tid; c < p.S; c += 32) M = fmax(M, static_cast<double>(__ldcg(p.part_max + r * p.S + c)));
-    for (int o = 16; o > 0; o >>= 1) M = fmax(M, __shfl_xor_sync(adt::kFullMask, M, o));
-    double sum = 0.0;
-    for (int c = tid; c < p.S; c += 32) {
-      const double mc = __ldcg(p.part_max + r * p.S + c);
-      sum += __ldcg(p.part_sum + r * p.S + c) * exp(mc - M);
+  // Pass 1: each thread's two largest values (ties kept).  Thread tid takes
+  // elements tid, tid + 256, ... of every tile.
+  float v1 = -INFINITY, v2 = -INFINITY;
+  for (int tt = 0; tt < ntiles; ++tt) {
+    const int t0 = c0 + tt * kTile, t1 = min(c1, t0 + kTile);
+    if (tt > 0) __syncthreads();  // the previous tile is consumed
+    ok &= stage_tile(vals, row, t0, t1, p, &s_bar, phase);
+#pragma unroll 8
+    for (int i = tid; i < t1 - t0; i += kThreads) {
+      const float x = vals[i];
+      v2 = fmaxf(v2, fminf(v1, x));
+      v1 = fmaxf(v1, x);
     }
-    sum = adt::warp_sum(sum);
-    if (tid == 0) s_lse = M + log(sum);
+  }
+  if (!ok && tid == 0) adt::raise_error(p.err, ADT_DEVERR_TIMEOUT);
+  // A warp's bound: a value with at least k of the warp's values at or above
+  // it: the k-th largest lane maximum (k <= 32), else the largest of the 64
+  // lane values (two per lane) with k of them at or above it.  The CTA's k
+  // best values are at or above the largest warp bound B.
+  {
+    float bw;
+    if (K <= 32) {
+      bw = warp_kth_largest(v1, K, lane);
+    } else {
+      int g1 = 0, g2 = 0;
+      for (int j = 0; j < 32; ++j) {
+        const float o1 = __shfl_sync(adt::kFullMask, v1, j), o2 = __shfl_sync(adt::kFullMask, v2, j);
+        g1 += (o1 >= v1) + (o2 >= v1);
+        g2 += (o1 >= v2) + (o2 >= v2);
+      }
+      float cb = -INFINITY;
+      if (g1 >= K) cb = v1;
+      if (g2 >= K) cb = fmaxf(cb, v2);
+      bw = adt::warp_max(cb);
+    }
+    const float mw = adt::warp_max(v1);
+    if (lane == 0) {
+      s_bw[warp] = bw;
+      s_mw[warp] = mw;
+    }
   }
   __syncthreads();
-  const double lse = s_lse;
-  const float ps = p.fscore[r];
-  const int32_t parent = p.fid ? p.fid[r] : r;
-  for (int j = tid; j < p.k; j += kThreads) {
-    const uint64_t key = sel[j];
-    const float x = adt::select_key_value(key);
-    const double lp = static_cast<double>(x) - lse;
-    const float score = static_cast<float>(static_cast<double>(ps) + lp);
-    const int64_t c = static_cast<int64_t>(r) * p.k + j;
+  float B = s_bw[0], M = s_mw[0];
+#pragma unroll
+  for (int w = 1; w < kWarps; ++w) {
+    B = fmaxf(B, s_bw[w]);
+    M = fmaxf(M, s_mw[w]);
+  }
+  // Pass 2: sum of exp(x - M) as 2^(x log2 e - M log2 e); gather the keys of
+  // values >= B (few: shared-memory atomics, no per-element vote).
+  const float Ml = M == -INFINITY ? 0.f : M * kLog2e;
+  float sa[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int tt = 0; tt < ntiles; ++tt) {
+    const int t0 = c0 + tt * kTile, t1 = min(c1, t0 + kTile);
+    if (ntiles > 1) {
+      __syncthreads();
+      ok &= stage_tile(vals, row, t0, t1, p, &s_bar, phase);
+    }
+    const int n = t1 - t0;
+    for (int i0 = tid; i0 < n; i0 += 4 * kThreads) {
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + u * kThreads;
+        if (i < n) {
+          const float x = vals[i];
+          sa[u] += ex2_approx(fmaf(x, kLog2e, -Ml));
+          if (x >= B) {
+            const unsigned pos = atomicAdd(&s_cnt, 1u);
+            if (pos < static_cast<unsigned>(kCandCap)) cand[pos] = adt::select_key(x, static_cast<uint32_t>(t0 + i));
+          }
+        }
+      }
+    }
+  }
+  {
+    const float sw = adt::warp_sum((sa[0] + sa[1]) + (sa[2] + sa[3]));
+    if (lane == 0) s_sw[warp] = sw;
+  }
+  __syncthreads();
+  const int cnt = static_cast<int>(s_cnt);
+  if (cnt <= kCandCap) {
+    rank_select(cand, cnt, K, ctl);
+  } else {
+    // Overflow (very many values at or above B): each warp keeps its k
+    // largest by insertion in a third pass, then the lists merge.
+    for (int i = tid; i < kWarps * kMaxK; i += kThreads) (&wl[0][0])[i] = 0ull;
+    const uint64_t kb = B == -INFINITY ? 1ull : adt::select_key(B, 0xffffffffu);  // lowest key of value B
+    WarpTopK tk;
+    uint64_t thr = 0ull;
+    for (int tt = 0; tt < ntiles; ++tt) {
+      const int t0 = c0 + tt * kTile, t1 = min(c1, t0 + kTile);
+      if (ntiles > 1) {
+        __syncthreads();
+        ok &= stage_tile(vals, row, t0, t1, p, &s_bar, phase);
+      }
+      const int n = t1 - t0;
+      for (int base = warp * 32; base < n; base += kThreads) {
+        const int i = base + lane;
+        const uint64_t key = i < n ? adt::select_key(vals[i], static_cast<uint32_t>(t0 + i)) : 0ull;
+        tk.offer(key >= kb ? key : 0ull, K, lane, thr);
+      }
+    }
+    __syncthreads();
+    wl[warp][lane] = tk.a;
+    wl[warp][lane + 32] = tk.b;
+    __syncthreads();
+    merge_topk(&wl[0][0], kWarps, kMaxK, K, K, ctl);
+  }
+  __syncthreads();
+  // This CTA's top k and (max, sum of exponentials), to the cluster's first CTA.
+  if (warp == 0) {
+    uint64_t* dst = cl.map_shared_rank(&cl_keys[rank * K], 0);
+    if (lane < K) dst[lane] = ctl[lane];
+    if (lane + 32 < K) dst[lane + 32] = ctl[lane + 32];
+    if (lane == 0) {
+      float S = 0.f;
+      for (int w = 0; w < kWarps; ++w) S += s_sw[w];
+      *cl.map_shared_rank(&cl_ms[rank], 0) = make_float2(M, S);
+    }
+  }
+  sm100::cluster_arrive_release();
+  sm100::cluster_wait_acquire();
+  if (rank != 0) return;
+
+  // ---- first CTA of row r: the row's top k and log-sum-exp, its children.
+  for (int i = tid; i < kMaxK; i += kThreads) rowl[i] = 0ull;
+  if (tid == 0) {
+    float Mr = -INFINITY, S = 0.f;
+    for (int c = 0; c < C; ++c) Mr = fmaxf(Mr, cl_ms[c].x);
+    for (int c = 0; c < C; ++c)
+      if (cl_ms[c].x != -INFINITY) S += cl_ms[c].y * ex2_approx((cl_ms[c].x - Mr) * kLog2e);
+    s_lse = static_cast<double>(Mr) + static_cast<double>(logf(S));
+  }
+  __syncthreads();
+  rank_select(cl_keys, C * K, K, rowl);
+  __syncthreads();
+  if (tid < K) {
+    const uint64_t key = rowl[tid];
+    const double lp = static_cast<double>(adt::select_key_value(key)) - s_lse;
+    const float score = static_cast<float>(static_cast<double>(p.fscore[r]) + lp);
+    const int64_t c = static_cast<int64_t>(r) * K + tid;
     p.ctok[c] = static_cast<int32_t>(adt::select_key_index(key));
     if (p.clogp) p.clogp[c] = static_cast<float>(lp);
     p.cscore[c] = score;
-    p.cpar[c] = parent;
+    p.cpar[c] = p.fid ? p.fid[r] : r;
     p.cross_keys[c] = adt::select_key(score, static_cast<uint32_t>(c));
   }
-  if (tid == 0) p.row_tickets[r] = 0u;
   __threadfence();
   __syncthreads();
   if (tid == 0) s_last = atomicAdd(p.all_ticket, 1u) == static_cast<unsigned>(p.F - 1);
@@ -157,38 +394,55 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
   __threadfence();
 
   // ---- last row: next frontier across all rows.
-  const int nc = p.F * p.k;
-  auto cross_key = [&](int i) { return __ldcg(p.cross_keys + i); };
-  const uint64_t thr3 = adt::block_topk_threshold<kThreads>(cross_key, nc, p.k_keep, &rs);
-  collect_sorted(cross_key, nc, thr3, p.k_keep, sel, &s_cnt);
-  for (int j = tid; j < p.k_keep; j += kThreads) {
-    const uint64_t key = sel[j];
-    const int32_t c = static_cast<int32_t>(adt::select_key_index(key));
-    p.keep[j] = c;
-    if (p.nscore) p.nscore[j] = adt::select_key_value(key);
-    if (p.nid) p.nid[j] = p.id_base + c;
+  const int nc = p.F * K;
+  if (p.k_keep <= kMaxK && nc <= kCandCap) {
+    for (int i = tid; i < nc; i += kThreads) cross_s[i] = __ldcg(p.cross_keys + i);
+    for (int i = tid; i < kMaxK; i += kThreads) rowl[i] = 0ull;
+    __syncthreads();
+    rank_select(cross_s, nc, p.k_keep, rowl);
+    __syncthreads();
+    if (tid < p.k_keep) {
+      const uint64_t key = rowl[tid];
+      const int32_t c = static_cast<int32_t>(adt::select_key_index(key));
+      p.keep[tid] = c;
+      if (p.nscore) p.nscore[tid] = adt::select_key_value(key);
+      if (p.nid) p.nid[tid] = p.id_base + c;
+    }
+  } else {
+    auto cross_key = [&](int i) { return __ldcg(p.cross_keys + i); };
+    const uint64_t thr3 = adt::block_topk_threshold<kThreads>(cross_key, nc, p.k_keep, &rs);
+    collect_sorted(cross_key, nc, thr3, p.k_keep, sel, &s_cnt);
+    for (int j = tid; j < p.k_keep; j += kThreads) {
+      const uint64_t key = sel[j];
+      const int32_t c = static_cast<int32_t>(adt::select_key_index(key));
+      p.keep[j] = c;
+      if (p.nscore) p.nscore[j] = adt::select_key_value(key);
+      if (p.nid) p.nid[j] = p.id_base + c;
+    }
   }
   if (tid == 0) *p.all_ticket = 0u;
 }
 
-// Workspace layout.  The completion counters sit at fixed offsets at the
-// start (room for the largest F), so calls of any shape can share one
-// workspace; the data regions after them are rewritten before being read.
+// CTAs per row (the cluster size).
+int expand_cluster(int V) {
+  const int c = (V + kValuesPerCta - 1) / kValuesPerCta;
+  return c < 1 ? 1 : (c > kMaxCluster ? kMaxCluster : c);
+}
+
+// Workspace layout.  The completion counter sits at a fixed offset at the
+// start, after a zeroed region kept for layout stability, so calls of any
+// shape can share one workspace; the keys after it are rewritten before use.
 constexpr int kMaxRows = 4096;
 
 struct ExpandWs {
-  size_t row_tickets, all_ticket, part_keys, part_max, part_sum, cross_keys, total;
+  size_t all_ticket, cross_keys, total;
 };
 
 ExpandWs expand_ws(int F, int V, int k) {
-  const size_t S = (static_cast<size_t>(V) + kChunk - 1) / kChunk;
+  (void)V;
   ExpandWs w{};
-  w.row_tickets = 0;
   w.all_ticket = kMaxRows * sizeof(unsigned);
-  w.part_keys = adt::align_up(w.all_ticket + sizeof(unsigned), 256);
-  w.part_max = adt::align_up(w.part_keys + F * S * k * sizeof(uint64_t), 256);
-  w.part_sum = adt::align_up(w.part_max + F * S * sizeof(float), 256);
-  w.cross_keys = adt::align_up(w.part_sum + F * S * sizeof(double), 256);
+  w.cross_keys = adt::align_up(w.all_ticket + sizeof(unsigned), 256);
   w.total = adt::align_up(w.cross_keys + static_cast<size_t>(F) * k * sizeof(uint64_t), 256);
   return w;
 }
@@ -333,7 +587,6 @@ adt_status adt_tree_expand(const float* logits, int64_t ld, const float* frontie
   p.V = V;
   p.k = k_child;
   p.k_keep = k_keep;
-  p.S = (V + kChunk - 1) / kChunk;
   p.T = temperature;
   p.use_T = temperature != 1.0f;
   p.id_base = child_id_base;
@@ -344,14 +597,33 @@ adt_status adt_tree_expand(const float* logits, int64_t ld, const float* frontie
   p.keep = keep_idx;
   p.nscore = next_score;
   p.nid = next_id;
-  p.part_keys = reinterpret_cast<uint64_t*>(ws + w.part_keys);
-  p.part_max = reinterpret_cast<float*>(ws + w.part_max);
-  p.part_sum = reinterpret_cast<double*>(ws + w.part_sum);
   p.cross_keys = reinterpret_cast<uint64_t*>(ws + w.cross_keys);
-  p.row_tickets = reinterpret_cast<unsigned*>(ws + w.row_tickets);
   p.all_ticket = reinterpret_cast<unsigned*>(ws + w.all_ticket);
-  dim3 grid(p.S, F);
-  expand_kernel<<<grid, kThreads, 0, adt::as_stream(stream)>>>(p);
+  p.err = info.error_word;
+  const int C = expand_cluster(V);
+  const int per = ((V + C - 1) / C + 3) & ~3;
+  const size_t dyn = static_cast<size_t>(per < kTile ? per : kTile) * sizeof(float);
+  static unsigned configured[2] = {0u, 0u};  // bit per device (< 64)
+  unsigned& word = configured[(info.device >> 5) & 1];
+  const unsigned bit = 1u << (info.device & 31);
+  if (!(__atomic_load_n(&word, __ATOMIC_ACQUIRE) & bit)) {
+    ADT_CUDA_TRY(cudaFuncSetAttribute(expand_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      static_cast<int>(kTile * sizeof(float))));
+    __atomic_fetch_or(&word, bit, __ATOMIC_ACQ_REL);
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.dynamicSmemBytes = dyn;
+  cfg.gridDim = dim3(static_cast<unsigned>(C), static_cast<unsigned>(F), 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.stream = adt::as_stream(stream);
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(C);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, expand_kernel, p));
   return adt::launch_status();
 }
 
