@@ -23,7 +23,7 @@ namespace cg = cooperative_groups;
 
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 1024;
 constexpr int kWarps = kThreads / 32;
 constexpr int kMaxK = 64;
 constexpr int kMaxKeep = 1024;
@@ -168,15 +168,15 @@ __device__ bool stage_tile(float* vals, const float* row, int t0, int t1, const 
 
 // out[rank] = key for the k largest of the n distinct nonzero keys in
 // keys[0..n) (0 entries skipped); out[] zeroed by the caller.  Block-wide:
-// every key counts the keys above it (broadcast reads, no dependent loads).
+// a warp takes a key and its lanes count the keys above it.
 __device__ void rank_select(const uint64_t* keys, int n, int k, uint64_t* out) {
-  for (int i = threadIdx.x; i < n; i += kThreads) {
+  const int lane = threadIdx.x & 31;
+  for (int i = threadIdx.x >> 5; i < n; i += kWarps) {
     const uint64_t key = keys[i];
     if (key == 0ull) continue;
     int rk = 0;
-#pragma unroll 8
-    for (int j = 0; j < n; ++j) rk += keys[j] > key;
-    if (rk < k) out[rk] = key;
+    for (int j = 0; j < n; j += 32) rk += __popc(__ballot_sync(adt::kFullMask, j + lane < n && keys[j + lane] > key));
+    if (lane == 0 && rk < k) out[rk] = key;
   }
 }
 
@@ -207,6 +207,7 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
   __shared__ uint64_t cand[kCandCap];              // keys at or above the CTA's bound
   __shared__ uint64_t wl[kWarps][kMaxK];           // overflow path: each warp's top k
   __shared__ float s_bw[kWarps], s_mw[kWarps], s_sw[kWarps];
+  __shared__ float s_B, s_M;
   __shared__ unsigned s_cnt;
   __shared__ uint64_t ctl[kMaxK];                  // this CTA's top k
   __shared__ uint64_t cl_keys[kMaxCluster * kMaxK];  // first CTA of the cluster: every CTA's k keys
@@ -254,15 +255,15 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
     }
   }
   if (!ok && tid == 0) adt::raise_error(p.err, ADT_DEVERR_TIMEOUT);
-  // A warp's bound: a value with at least k of the warp's values at or above
-  // it: the k-th largest lane maximum (k <= 32), else the largest of the 64
-  // lane values (two per lane) with k of them at or above it.  The CTA's k
-  // best values are at or above the largest warp bound B.
+  // The bound B: a value with at least k of the CTA's logits at or above it,
+  // so that its k best are among those >= B.  For k <= 32: the k-th largest
+  // of the 32 warp maxima (one bitonic sort in warp 0).  For larger k: per
+  // warp, the largest of its 64 lane values (two per lane) with k of them at
+  // or above it; B is the largest of those.
   {
-    float bw;
-    if (K <= 32) {
-      bw = warp_kth_largest(v1, K, lane);
-    } else {
+    const float mw = adt::warp_max(v1);
+    float bw = -INFINITY;
+    if (K > 32) {
       int g1 = 0, g2 = 0;
       for (int j = 0; j < 32; ++j) {
         const float o1 = __shfl_sync(adt::kFullMask, v1, j), o2 = __shfl_sync(adt::kFullMask, v2, j);
@@ -274,19 +275,23 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
       if (g2 >= K) cb = fmaxf(cb, v2);
       bw = adt::warp_max(cb);
     }
-    const float mw = adt::warp_max(v1);
     if (lane == 0) {
       s_bw[warp] = bw;
       s_mw[warp] = mw;
     }
   }
   __syncthreads();
-  float B = s_bw[0], M = s_mw[0];
-#pragma unroll
-  for (int w = 1; w < kWarps; ++w) {
-    B = fmaxf(B, s_bw[w]);
-    M = fmaxf(M, s_mw[w]);
+  if (warp == 0) {
+    const float mv = s_mw[lane];
+    const float mmax = adt::warp_max(mv);
+    const float b = K <= 32 ? warp_kth_largest(mv, K, lane) : adt::warp_max(s_bw[lane]);
+    if (lane == 0) {
+      s_B = b;
+      s_M = mmax;
+    }
   }
+  __syncthreads();
+  const float B = s_B, M = s_M;
   // Pass 2: sum of exp(x - M) as 2^(x log2 e - M log2 e); gather the keys of
   // values >= B (few: shared-memory atomics, no per-element vote).
   const float Ml = M == -INFINITY ? 0.f : M * kLog2e;
