@@ -285,6 +285,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int g = h / p.group;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
+  // Programmatic dependent launch: every global-memory access comes after
+  // the previous kernel in the stream has completed (immediate when this
+  // launch does not overlap one).
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
   const int node0 = p.offs[b];
   const int n = p.offs[b + 1] - node0;
   const int total_nodes = p.offs[p.B];
@@ -659,6 +663,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   // ------------------------------------------------------------ epilogue
+  // The next kernel in the stream may start its set-up now.
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
   // The softmax threads take their rows of O (unnormalised) into registers.
   constexpr int kOB = D / 64;
   uint32_t o[kOB][32];
@@ -984,7 +990,7 @@ int max_active_clusters(int D, int cluster, int dev) {
 
 template <int D>
 adt_status launch(TcParams prm, const void* k_cache, const void* v_cache, int64_t sb, int64_t sh, cudaStream_t st,
-                  int dev) {
+                  int dev, bool overlap_previous) {
   static unsigned configured[2] = {0u, 0u};  // bit per device (< 64)
   const unsigned bit = 1u << (dev & 31);
   unsigned& word = configured[dev >> 5];
@@ -1004,13 +1010,17 @@ adt_status launch(TcParams prm, const void* k_cache, const void* v_cache, int64_
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = Cfg<D>::kDynSmem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = prm.cluster_merge ? static_cast<unsigned>(prm.splits) : 1u;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  // Programmatic dependent launch: the launch and the set-up before the
+  // kernel's griddepcontrol.wait may overlap the tail of the previous kernel.
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = overlap_previous ? 2 : 1;
   ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, tree_attn_tc_kernel<D>, tm_k, tm_v, prm));
   return adt::launch_status();
 }
@@ -1093,8 +1103,8 @@ adt_status adt_tree_attn(const adt_bf16* q, const adt_bf16* k_cache, const adt_b
   prm.part_ml = reinterpret_cast<float2*>(ws + w.part_ml);
   prm.tickets = reinterpret_cast<unsigned*>(ws + w.tickets);
   cudaStream_t s = adt::as_stream(stream);
-  return D == 128 ? launch<128>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device)
-                  : launch<64>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device);
+  return D == 128 ? launch<128>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device, true)
+                  : launch<64>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device, true);
 }
 
 }  // extern "C"
@@ -1179,6 +1189,6 @@ extern "C" adt_status adt_tree_attn_noalloc(const adt_bf16* q, const adt_bf16* k
   prm.part_o = reinterpret_cast<float*>(ws + w.part_o);
   prm.part_ml = reinterpret_cast<float2*>(ws + w.part_ml);
   prm.tickets = reinterpret_cast<unsigned*>(ws + w.tickets);
-  return D == 128 ? launch<128>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device)
-                  : launch<64>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device);
+  return D == 128 ? launch<128>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device, false)
+                  : launch<64>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device, false);
 }
