@@ -151,7 +151,7 @@ def run_gpu(args, wl, rank, world):
     mode = {"greedy": B.ACCEPT_GREEDY, "spec_det": B.ACCEPT_SPEC_DET}[args.mode]
     shape = StepShape(layers=wl["layers"], H=wl["H"], Hkv=wl["Hkv"], D=wl["D"], V=wl["V"], kv_len=wl["kv_len"],
                       depth=wl["depth"], width=wl["width"], max_nodes=wl["max_nodes"], mode=mode, temperature=1.0)
-    step = TreeVerifyStep(shape)
+    step = TreeVerifyStep(shape, input_slots=2)
     fill_inputs_on_device(step, 20251221 + rank)
     stream = torch.cuda.Stream()
     torch.cuda.synchronize()
@@ -217,30 +217,77 @@ def run_gpu(args, wl, rank, world):
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         step_ms = float(t.item())
 
-    # end to end through the public API: per-step inputs copied from pinned
-    # host memory, results read back, host synchronised every step
-    per_step_inputs = [step.q, step.k_tree, step.v_tree, step.target, step.u_accept, step.u_sample,
-                       step.root_token] + list(step.draft_rows)
-    host_in = [t.cpu().pin_memory() for t in per_step_inputs]
+    # End to end through the public API: every step copies its inputs from
+    # pinned host memory into one of two input slots and reads its result
+    # back; the copy of step i + 1 (its own stream) overlaps the compute of
+    # step i, as a serving loop would run it.
+    step.use_slot(1)
+    for name in step.STEP_INPUTS:
+        src = getattr(step, "_slots")[0][name]
+        dst = getattr(step, name)
+        if isinstance(src, list):
+            for a, b_ in zip(dst, src):
+                a.copy_(b_)
+        else:
+            dst.copy_(src)
+    graphs1 = [torch.cuda.CUDAGraph() for _ in range(3)]
+    with torch.cuda.stream(stream):
+        with torch.cuda.graph(graphs1[0], stream=stream):
+            step.launch_draft(stream)
+        with torch.cuda.graph(graphs1[1], stream=stream):
+            for layer in range(shape.layers):
+                step.launch_attention(layer, stream)
+        with torch.cuda.graph(graphs1[2], stream=stream):
+            step.launch_verify(stream)
+    step.use_slot(0)
+    torch.cuda.synchronize()
+    slot_graphs = [graphs, graphs1]
+    slot_inputs = []
+    for i in range(2):
+        step.use_slot(i)
+        slot_inputs.append(step.step_input_tensors())
+    step.use_slot(0)
+    host_in = [t.cpu().pin_memory() for t in slot_inputs[0]]
     outputs = [step.path, step.accept_len, step.bonus, step.kv_len_out]
-    host_out = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in outputs]
+    host_out = [[torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in outputs] for _ in range(2)]
     h2d = sum(t.numel() * t.element_size() for t in host_in)
-    d2h = sum(t.numel() * t.element_size() for t in host_out)
+    d2h = sum(t.numel() * t.element_size() for t in host_out[0])
+    copy_stream = torch.cuda.Stream()
+    copied = [torch.cuda.Event() for _ in range(2)]
+    consumed = [torch.cuda.Event() for _ in range(2)]
+    done = [torch.cuda.Event() for _ in range(2)]
+
+    def issue(i):
+        sl = i % 2
+        if i >= 2:
+            copy_stream.wait_event(consumed[sl])
+        with torch.cuda.stream(copy_stream):
+            for d, h in zip(slot_inputs[sl], host_in):
+                d.copy_(h, non_blocking=True)
+            copied[sl].record(copy_stream)
+        stream.wait_event(copied[sl])
+        with torch.cuda.stream(stream):
+            for gr in slot_graphs[sl]:
+                gr.replay()
+            consumed[sl].record(stream)
+            for h, d in zip(host_out[sl], outputs):
+                h.copy_(d, non_blocking=True)
+            done[sl].record(stream)
+
     K2 = max(3, min(K, args.e2e_steps))
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    with torch.cuda.stream(stream):
-        e0.record(stream)
-        for _ in range(K2):
-            for d, h in zip(per_step_inputs, host_in):
-                d.copy_(h, non_blocking=True)
-            one_step()
-            for h, d in zip(host_out, outputs):
-                h.copy_(d, non_blocking=True)
-            stream.synchronize()
-        e1.record(stream)
+    e0.record(stream)
+    copy_stream.wait_event(e0)
+    issue(0)
+    for i in range(K2):
+        if i + 1 < K2:
+            issue(i + 1)
+        done[i % 2].synchronize()
+        _ = int(host_out[i % 2][1][0])  # the host reads step i's result
+    e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1) / K2
     if world > 1:

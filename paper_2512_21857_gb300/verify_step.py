@@ -53,7 +53,11 @@ class StepShape:
 class TreeVerifyStep:
     """Persistent buffers and the launch sequence of one verify step."""
 
-    def __init__(self, shape: StepShape, device="cuda", keep_layer_outputs=False):
+    # Per-step inputs (what the model produces for each step); the KV cache
+    # persists across steps.
+    STEP_INPUTS = ("q", "k_tree", "v_tree", "target", "u_accept", "u_sample", "root_token", "draft_rows")
+
+    def __init__(self, shape: StepShape, device="cuda", keep_layer_outputs=False, input_slots=1):
         s = self.shape = shape
         self.device = device
         Bn = s.batch
@@ -71,14 +75,18 @@ class TreeVerifyStep:
         # model-side tensors (inputs of the step)
         self.k_cache = torch.zeros((s.layers, Bn, s.Hkv, self.lmax, s.D), **bf16)
         self.v_cache = torch.zeros((s.layers, Bn, s.Hkv, self.lmax, s.D), **bf16)
-        self.q = torch.zeros((s.layers, self.ntot, s.H, s.D), **bf16)
-        self.k_tree = torch.zeros((s.layers, self.ntot, s.Hkv, s.D), **bf16)
-        self.v_tree = torch.zeros((s.layers, self.ntot, s.Hkv, s.D), **bf16)
-        self.draft_rows = [torch.zeros((s.depth[b], s.width[b], s.V), **f32) for b in range(Bn)]
-        self.target = torch.zeros((self.ntot, s.V), **f32)
-        self.u_accept = torch.zeros(self.ntot, **f32)
-        self.u_sample = torch.zeros(self.ntot, **f32)
-        self.root_token = torch.zeros(Bn, **i32)
+        # per-step inputs: `input_slots` copies, so that the inputs of the next
+        # step can be copied in while this one computes (use_slot picks one)
+        self._slots = [dict(q=torch.zeros((s.layers, self.ntot, s.H, s.D), **bf16),
+                            k_tree=torch.zeros((s.layers, self.ntot, s.Hkv, s.D), **bf16),
+                            v_tree=torch.zeros((s.layers, self.ntot, s.Hkv, s.D), **bf16),
+                            draft_rows=[torch.zeros((s.depth[b], s.width[b], s.V), **f32) for b in range(Bn)],
+                            target=torch.zeros((self.ntot, s.V), **f32),
+                            u_accept=torch.zeros(self.ntot, **f32),
+                            u_sample=torch.zeros(self.ntot, **f32),
+                            root_token=torch.zeros(Bn, **i32))
+                       for _ in range(input_slots)]
+        self.use_slot(0)
         self.kv_len = torch.tensor(s.kv_len, **i32)
         self.node_offsets = torch.tensor(offs, **i32)
         # intermediate and output buffers
@@ -109,6 +117,18 @@ class TreeVerifyStep:
                                                 for b in range(Bn)), dev)
         self.ws_attn = B.zeroed_workspace(
             B.adt_tree_attn_workspace_size(Bn, s.H, s.D, s.max_nodes, self.lmax), dev)
+
+    def use_slot(self, i):
+        """Points the step's per-step input attributes at input slot i; the
+        launches that follow (and graphs captured from them) read that slot."""
+        self.slot = i
+        for name, t in self._slots[i].items():
+            setattr(self, name, t)
+
+    def step_input_tensors(self):
+        """The current slot's per-step input tensors, in a fixed order."""
+        return [self.q, self.k_tree, self.v_tree, self.target, self.u_accept, self.u_sample,
+                self.root_token] + list(self.draft_rows)
 
     # -------------------------------------------------------------- phases
     def launch_draft(self, stream=None):
