@@ -124,6 +124,20 @@ def tree_attention(q, k_cache, v_cache, kv_len, k_tree, v_tree, parents, node_of
 # EAGLE-2 node score, Eq. 4)
 # ----------------------------------------------------------------------------
 
+def cfg_logits(cond, uncond, scale: float) -> np.ndarray:
+    """Classifier-free guidance on logits.  The paper computes both p and q
+    under CFG (Sec. 3.1, under Eq. 1) with guidance scale 3.0 (Sec. 5.1) but
+    prints no formula; the standard combine is taken:
+        l = l_uncond + s * (l_cond - l_uncond),
+    each operation (difference, product, sum) rounded to fp32 as written.
+    The result then goes through the usual definitions (expansion, walk)."""
+    c = np.asarray(cond, dtype=np.float32)
+    u = np.asarray(uncond, dtype=np.float32)
+    s = np.float32(scale)
+    d = (c - u).astype(np.float32)
+    return (u + (s * d).astype(np.float32)).astype(np.float32)
+
+
 def _tempered(row32, temperature: float) -> np.ndarray:
     """Row / T in fp32 (the stored type), -0.0 canonicalised to +0.0."""
     x = np.asarray(row32, dtype=np.float32)
