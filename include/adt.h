@@ -202,6 +202,28 @@ adt_status adt_tree_expand(const float* logits, int64_t ld, const float* frontie
                            void* stream);
 
 /* ------------------------------------------------------------------------
+ * adt_tree_expand_cfg - adt_tree_expand on classifier-free-guided logits.
+ * The paper computes the draft distribution q under classifier-free guidance
+ * (Sec. 3.1, the sentence under Eq. 1; Fig. 5's conditional and
+ * unconditional draft branches) with guidance scale 3.0 (Sec. 5.1).  Row r's
+ * logits are formed on the fly from the two branches,
+ *     l = uncond + cfg_scale * (cond - uncond),
+ * each operation rounded to fp32 as written, then divided by temperature;
+ * everything else is adt_tree_expand.
+ *
+ * logits_cond, logits_uncond [device] fp32, row r at + r*ld, same ld, both
+ *         16-byte aligned; cfg_scale finite.  Other arguments and the
+ *         workspace as for adt_tree_expand (one workspace serves both).
+ * ------------------------------------------------------------------------ */
+adt_status adt_tree_expand_cfg(const float* logits_cond, const float* logits_uncond, int64_t ld,
+                               float cfg_scale, const float* frontier_score, const int32_t* frontier_id,
+                               int32_t F, int32_t V, int32_t k_child, int32_t k_keep, float temperature,
+                               int32_t child_id_base, int32_t* child_token, float* child_logp,
+                               float* child_score, int32_t* child_parent, int32_t* keep_idx,
+                               float* next_score, int32_t* next_id, void* workspace,
+                               size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
  * adt_tree_rerank - the final draft tree (Eq. 4 and the sentence after it:
  * the top-N nodes by score form the tree that the target verifies).
  *
@@ -263,6 +285,29 @@ adt_status adt_tree_accept(const float* target_logits, int64_t ld_target,
                            float temperature, int32_t* path, int32_t max_path,
                            int32_t* accept_len, int32_t* bonus_token, void* workspace,
                            size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * adt_tree_accept_cfg - adt_tree_accept with p and q computed under
+ * classifier-free guidance (Sec. 3.1, the sentence under Eq. 1; guidance
+ * scale 3.0 in Sec. 5.1).  Every target (and, in SPEC mode, draft) row is
+ * formed on the fly as uncond + cfg_scale * (cond - uncond), each operation
+ * rounded to fp32 as written, before the division by temperature; the walk
+ * is that of adt_tree_accept.
+ *
+ * target_cond, target_uncond [device] fp32, same layout and ld_target.
+ * draft_cond, draft_uncond   [device] fp32, same layout and ld_draft (SPEC
+ *         mode only, else may be NULL); draft_row maps nodes to rows as in
+ *         adt_tree_accept.  cfg_scale finite.  Other arguments as for
+ *         adt_tree_accept.
+ * ------------------------------------------------------------------------ */
+adt_status adt_tree_accept_cfg(const float* target_cond, const float* target_uncond, int64_t ld_target,
+                               const float* draft_cond, const float* draft_uncond, int64_t ld_draft,
+                               const int32_t* draft_row, float cfg_scale, const int32_t* tokens,
+                               const int32_t* parents, const int32_t* node_offsets, int32_t B, int32_t V,
+                               int32_t max_nodes, const float* u_accept, const float* u_sample,
+                               adt_accept_mode mode, float temperature, int32_t* path, int32_t max_path,
+                               int32_t* accept_len, int32_t* bonus_token, void* workspace,
+                               size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
  * adt_kv_compact - commit the accepted path to the KV cache, all layers in

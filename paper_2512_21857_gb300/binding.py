@@ -26,9 +26,9 @@ DEVERR_BAD_TREE, DEVERR_KV_RANGE, DEVERR_BAD_PATH, DEVERR_TIMEOUT, DEVERR_BAD_IN
 EXPORTED = [
     "adt_version", "adt_get_device_error", "adt_status_string",
     "adt_tree_attn_workspace_size", "adt_tree_attn", "adt_tree_attn_noalloc",
-    "adt_tree_expand_workspace_size", "adt_tree_expand",
+    "adt_tree_expand_workspace_size", "adt_tree_expand", "adt_tree_expand_cfg",
     "adt_tree_rerank_workspace_size", "adt_tree_rerank",
-    "adt_tree_accept_workspace_size", "adt_tree_accept",
+    "adt_tree_accept_workspace_size", "adt_tree_accept", "adt_tree_accept_cfg",
     "adt_kv_compact",
     "adt_ctrl_create", "adt_ctrl_destroy", "adt_ctrl_next", "adt_ctrl_update", "adt_ctrl_get",
 ]
@@ -61,11 +61,15 @@ _SIGS = {
     "adt_tree_expand_workspace_size": ([_I32] * 3, _SZ),
     "adt_tree_expand": ([_P, _I64, _P, _P, _I32, _I32, _I32, _I32, _F32, _I32, _P, _P, _P, _P, _P, _P, _P,
                          _P, _SZ, _P], _I32),
+    "adt_tree_expand_cfg": ([_P, _P, _I64, _F32, _P, _P, _I32, _I32, _I32, _I32, _F32, _I32, _P, _P, _P, _P, _P,
+                             _P, _P, _P, _SZ, _P], _I32),
     "adt_tree_rerank_workspace_size": ([_I32], _SZ),
     "adt_tree_rerank": ([_P, _P, _P, _I32, _P, _I32, _P, _P, _P, _P, _P, _SZ, _P], _I32),
     "adt_tree_accept_workspace_size": ([_I32, _I32], _SZ),
     "adt_tree_accept": ([_P, _I64, _P, _I64, _P, _P, _P, _P, _I32, _I32, _I32, _P, _P, _I32, _F32, _P, _I32,
                          _P, _P, _P, _SZ, _P], _I32),
+    "adt_tree_accept_cfg": ([_P, _P, _I64, _P, _P, _I64, _P, _F32, _P, _P, _P, _I32, _I32, _I32, _P, _P, _I32,
+                             _F32, _P, _I32, _P, _P, _P, _SZ, _P], _I32),
     "adt_kv_compact": ([_P, _P, _P, _P, _P, _P, _P, _P, _I32, _P, _I32, _I32, _I32, _I32, _I32, _I64, _I64,
                         _I64, _I64, _P], _I32),
     "adt_ctrl_create": ([ctypes.POINTER(CtrlParams), _I32, _I32, ctypes.POINTER(_P)], _I32),
@@ -194,6 +198,25 @@ def adt_tree_expand(logits, frontier_score, frontier_id, *, F, V, k_child, k_kee
     _check(st, "adt_tree_expand")
 
 
+def adt_tree_expand_cfg(logits_cond, logits_uncond, frontier_score, frontier_id, *, cfg_scale, F, V, k_child,
+                        k_keep, temperature=1.0, child_id_base=0, child_token, child_logp, child_score,
+                        child_parent, keep_idx, next_score=None, next_id=None, workspace, stream=None) -> None:
+    """adt_tree_expand on uncond + cfg_scale * (cond - uncond); both [F, V] rows share one row stride."""
+    _expect(frontier_score, torch.float32, "frontier_score")
+    for t in (logits_cond, logits_uncond):
+        if t.dtype != torch.float32 or t.dim() != 2 or t.stride(-1) != 1:
+            raise TypeError("logits: fp32 [F, V] rows with unit inner stride")
+    if logits_cond.stride(0) != logits_uncond.stride(0):
+        raise ValueError("conditional and unconditional rows must share a row stride")
+    st = lib().adt_tree_expand_cfg(_ptr(logits_cond), _ptr(logits_uncond), logits_cond.stride(0), float(cfg_scale),
+                                   _ptr(frontier_score), _ptr(frontier_id), F, V, k_child, k_keep,
+                                   float(temperature), int(child_id_base), _ptr(child_token), _ptr(child_logp),
+                                   _ptr(child_score), _ptr(child_parent), _ptr(keep_idx), _ptr(next_score),
+                                   _ptr(next_id), _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                   _stream(stream))
+    _check(st, "adt_tree_expand_cfg")
+
+
 def adt_tree_rerank(cand_token, cand_score, cand_parent, C, root_token, n_nodes, *, tokens, parents,
                     cand_index=None, depth=None, workspace, stream=None) -> None:
     st = lib().adt_tree_rerank(_ptr(cand_token), _ptr(cand_score), _ptr(cand_parent), int(C), _ptr(root_token),
@@ -214,6 +237,23 @@ def adt_tree_accept(target_logits, draft_logits, tokens, parents, node_offsets, 
                                _ptr(accept_len), _ptr(bonus_token), _ptr(ws),
                                0 if ws is None else ws.numel() * ws.element_size(), _stream(stream))
     _check(st, "adt_tree_accept")
+
+
+def adt_tree_accept_cfg(target_cond, target_uncond, draft_cond, draft_uncond, tokens, parents, node_offsets, *,
+                        cfg_scale, B, V, max_nodes, mode, u_accept=None, u_sample=None, temperature=1.0, path,
+                        max_path, accept_len, bonus_token, draft_row=None, stream=None) -> None:
+    """adt_tree_accept with every target / draft row formed as uncond + cfg_scale * (cond - uncond)."""
+    if target_cond.stride(0) != target_uncond.stride(0):
+        raise ValueError("conditional and unconditional target rows must share a row stride")
+    ldd = draft_cond.stride(0) if draft_cond is not None else 0
+    if draft_cond is not None and draft_uncond is not None and draft_uncond.stride(0) != ldd:
+        raise ValueError("conditional and unconditional draft rows must share a row stride")
+    st = lib().adt_tree_accept_cfg(_ptr(target_cond), _ptr(target_uncond), target_cond.stride(0), _ptr(draft_cond),
+                                   _ptr(draft_uncond), ldd, _ptr(draft_row), float(cfg_scale), _ptr(tokens),
+                                   _ptr(parents), _ptr(node_offsets), B, V, max_nodes, _ptr(u_accept),
+                                   _ptr(u_sample), int(mode), float(temperature), _ptr(path), int(max_path),
+                                   _ptr(accept_len), _ptr(bonus_token), None, 0, _stream(stream))
+    _check(st, "adt_tree_accept_cfg")
 
 
 def adt_kv_compact(k_cache, v_cache, kv_len, kv_len_out, k_tree, v_tree, node_offsets, path, max_path,

@@ -48,6 +48,13 @@ __device__ __forceinline__ void raise_error(unsigned* word, unsigned bits) {
   if (word) atomicOr(word, bits);
 }
 
+// Classifier-free guidance on one logit: u + s (c - u), each operation
+// rounded to fp32 as written (no contraction), so that the selections made
+// on the result match a reference that rounds the same way.
+__device__ __forceinline__ float cfg_combine(float c, float u, float s) {
+  return __fadd_rn(u, __fmul_rn(s, __fsub_rn(c, u)));
+}
+
 // Order-preserving map of a finite float to uint32 (larger float -> larger
 // key); -0.0 and +0.0 map to the same key.
 __device__ __forceinline__ uint32_t float_order_key(float f) {

@@ -29,6 +29,9 @@ struct AcceptParams {
   int64_t ldt;
   const float* draft;
   int64_t ldd;
+  const float* target_u;  // classifier-free guidance: unconditional rows (same layout), else NULL
+  const float* draft_u;
+  float cfg;              // guidance scale
   const int32_t* drow;
   const int32_t* tokens;
   const int32_t* parents;
@@ -117,16 +120,28 @@ __device__ void block_argmax(float& v, int& idx, Shared* sh) {
   }
 }
 
-// Loads this CTA's slice of a logit row (divided by T) into buf; entries
-// past V are -inf.
-__device__ void load_slice(const float* row, int lo, int cnt, int Vs, float* buf, const AcceptParams& p) {
+// Loads this CTA's slice of a logit row (under guidance u + s (c - u) with
+// the unconditional row row_u; then divided by T) into buf; entries past V
+// are -inf.
+__device__ void load_slice(const float* row, const float* row_u, int lo, int cnt, int Vs, float* buf,
+                           const AcceptParams& p) {
   for (int i = threadIdx.x * 4; i < Vs; i += kThreads * 4) {
     float x[4];
     if (i + 3 < cnt) {
       const float4 v = __ldg(reinterpret_cast<const float4*>(row + lo + i));
       x[0] = v.x; x[1] = v.y; x[2] = v.z; x[3] = v.w;
+      if (row_u) {
+        const float4 w = __ldg(reinterpret_cast<const float4*>(row_u + lo + i));
+        x[0] = adt::cfg_combine(x[0], w.x, p.cfg);
+        x[1] = adt::cfg_combine(x[1], w.y, p.cfg);
+        x[2] = adt::cfg_combine(x[2], w.z, p.cfg);
+        x[3] = adt::cfg_combine(x[3], w.w, p.cfg);
+      }
     } else {
-      for (int e = 0; e < 4; ++e) x[e] = (i + e < cnt) ? __ldg(row + lo + i + e) : -INFINITY;
+      for (int e = 0; e < 4; ++e)
+        x[e] = (i + e < cnt) ? (row_u ? adt::cfg_combine(__ldg(row + lo + i + e), __ldg(row_u + lo + i + e), p.cfg)
+                                      : __ldg(row + lo + i + e))
+                             : -INFINITY;
     }
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
@@ -297,12 +312,14 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
     const int nk = sh.nkids;
     const int gv = node0 + v;
     const float* trow = p.target + static_cast<int64_t>(gv) * p.ldt;
+    const float* trow_u = p.target_u ? p.target_u + static_cast<int64_t>(gv) * p.ldt : nullptr;
 
     if (p.mode == ADT_ACCEPT_GREEDY) {
       float bv = -INFINITY;
       int bi = 0x7fffffff;
       for (int i = tid; i < cnt; i += kThreads) {
-        const float x = __ldg(trow + lo + i);
+        float x = __ldg(trow + lo + i);
+        if (trow_u) x = adt::cfg_combine(x, __ldg(trow_u + lo + i), p.cfg);
         if (better(x, lo + i, bv, bi)) {
           bv = x;
           bi = lo + i;
@@ -344,10 +361,10 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
     // ---- sampling modes: p = softmax(target row / T) in the slices.
     const bool spec = p.mode == ADT_ACCEPT_SPEC;
     const bool need_q = spec && nk > 0;
-    load_slice(trow, lo, cnt, p.Vs, pbuf, p);
+    load_slice(trow, trow_u, lo, cnt, p.Vs, pbuf, p);
     if (need_q) {
       const int64_t dr = p.drow ? p.drow[gv] : gv;
-      load_slice(p.draft + dr * p.ldd, lo, cnt, p.Vs, qbuf, p);
+      load_slice(p.draft + dr * p.ldd, p.draft_u ? p.draft_u + dr * p.ldd : nullptr, lo, cnt, p.Vs, qbuf, p);
     }
     __syncthreads();
     const float mp = slice_max(pbuf, p.Vs, &sh);
@@ -492,22 +509,14 @@ int slice_for(int V, int cs) {
 
 }  // namespace
 
-extern "C" {
-
-size_t adt_tree_accept_workspace_size(int32_t B, int32_t V) {
-  (void)B;
-  (void)V;
-  return 0;
-}
-
-adt_status adt_tree_accept(const float* target_logits, int64_t ld_target,
-                           const float* draft_logits, int64_t ld_draft, const int32_t* draft_row,
-                           const int32_t* tokens, const int32_t* parents,
-                           const int32_t* node_offsets, int32_t B, int32_t V, int32_t max_nodes,
-                           const float* u_accept, const float* u_sample, adt_accept_mode mode,
-                           float temperature, int32_t* path, int32_t max_path,
-                           int32_t* accept_len, int32_t* bonus_token, void* workspace,
-                           size_t workspace_bytes, void* stream) {
+static adt_status accept_impl(const float* target_logits, const float* target_u, int64_t ld_target,
+                              const float* draft_logits, const float* draft_u, int64_t ld_draft,
+                              const int32_t* draft_row, float cfg_scale, const int32_t* tokens,
+                              const int32_t* parents, const int32_t* node_offsets, int32_t B, int32_t V,
+                              int32_t max_nodes, const float* u_accept, const float* u_sample,
+                              adt_accept_mode mode, float temperature, int32_t* path, int32_t max_path,
+                              int32_t* accept_len, int32_t* bonus_token, void* workspace,
+                              size_t workspace_bytes, void* stream) {
   (void)workspace;
   (void)workspace_bytes;
   ADT_REQUIRE(target_logits && tokens && parents && node_offsets && path && accept_len && bonus_token);
@@ -521,6 +530,10 @@ adt_status adt_tree_accept(const float* target_logits, int64_t ld_target,
   }
   if (mode == ADT_ACCEPT_SPEC) {
     ADT_REQUIRE(draft_logits && ld_draft >= V && ld_draft % 4 == 0 && adt::aligned16(draft_logits));
+  }
+  if (target_u) {
+    ADT_REQUIRE(adt::aligned16(target_u) && cfg_scale > -1e30f && cfg_scale < 1e30f);
+    if (mode == ADT_ACCEPT_SPEC) ADT_REQUIRE(draft_u && adt::aligned16(draft_u));
   }
   adt::DeviceInfo info;
   adt_status st = adt::device_info(&info);
@@ -547,6 +560,9 @@ adt_status adt_tree_accept(const float* target_logits, int64_t ld_target,
   p.draft = draft_logits;
   p.ldd = ld_draft;
   p.drow = draft_row;
+  p.target_u = target_u;
+  p.draft_u = target_u ? draft_u : nullptr;
+  p.cfg = cfg_scale;
   p.tokens = tokens;
   p.parents = parents;
   p.offs = node_offsets;
@@ -579,6 +595,41 @@ adt_status adt_tree_accept(const float* target_logits, int64_t ld_target,
   cfg.numAttrs = 1;
   ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, accept_kernel, p));
   return adt::launch_status();
+}
+
+extern "C" {
+
+size_t adt_tree_accept_workspace_size(int32_t B, int32_t V) {
+  (void)B;
+  (void)V;
+  return 0;
+}
+
+adt_status adt_tree_accept(const float* target_logits, int64_t ld_target,
+                           const float* draft_logits, int64_t ld_draft, const int32_t* draft_row,
+                           const int32_t* tokens, const int32_t* parents,
+                           const int32_t* node_offsets, int32_t B, int32_t V, int32_t max_nodes,
+                           const float* u_accept, const float* u_sample, adt_accept_mode mode,
+                           float temperature, int32_t* path, int32_t max_path,
+                           int32_t* accept_len, int32_t* bonus_token, void* workspace,
+                           size_t workspace_bytes, void* stream) {
+  return accept_impl(target_logits, nullptr, ld_target, draft_logits, nullptr, ld_draft, draft_row, 0.f, tokens,
+                     parents, node_offsets, B, V, max_nodes, u_accept, u_sample, mode, temperature, path, max_path,
+                     accept_len, bonus_token, workspace, workspace_bytes, stream);
+}
+
+adt_status adt_tree_accept_cfg(const float* target_cond, const float* target_uncond, int64_t ld_target,
+                               const float* draft_cond, const float* draft_uncond, int64_t ld_draft,
+                               const int32_t* draft_row, float cfg_scale, const int32_t* tokens,
+                               const int32_t* parents, const int32_t* node_offsets, int32_t B, int32_t V,
+                               int32_t max_nodes, const float* u_accept, const float* u_sample,
+                               adt_accept_mode mode, float temperature, int32_t* path, int32_t max_path,
+                               int32_t* accept_len, int32_t* bonus_token, void* workspace,
+                               size_t workspace_bytes, void* stream) {
+  ADT_REQUIRE(target_uncond);
+  return accept_impl(target_cond, target_uncond, ld_target, draft_cond, draft_uncond, ld_draft, draft_row,
+                     cfg_scale, tokens, parents, node_offsets, B, V, max_nodes, u_accept, u_sample, mode,
+                     temperature, path, max_path, accept_len, bonus_token, workspace, workspace_bytes, stream);
 }
 
 }  // extern "C"

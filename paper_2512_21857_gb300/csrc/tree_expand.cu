@@ -36,6 +36,8 @@ constexpr float kLog2e = 1.44269504088896340736f;
 
 struct ExpandParams {
   const float* logits;
+  const float* logits_u;  // classifier-free guidance: unconditional rows (same ld), else NULL
+  float cfg;              // guidance scale
   int64_t ld;
   const float* fscore;
   const int32_t* fid;
@@ -140,27 +142,40 @@ struct WarpTopK {
 };
 
 // Stages logits [t0, t1) of a row (t0 a multiple of 4; rows start 16-byte
-// aligned and ld is a multiple of 4) in shared memory with one bulk copy,
-// waiting with a bound.  Then divides by the temperature in place.  Block-wide.
-__device__ bool stage_tile(float* vals, const float* row, int t0, int t1, const ExpandParams& p, uint64_t* bar,
-                           uint32_t& phase) {
+// aligned and ld is a multiple of 4) in shared memory with one bulk copy
+// (two with guidance: the unconditional row goes to vals_u), waiting with a
+// bound; then forms u + s (c - u) under guidance and divides by the
+// temperature, in place.  Block-wide.
+__device__ bool stage_tile(float* vals, float* vals_u, const float* row, const float* row_u, int t0, int t1,
+                           const ExpandParams& p, uint64_t* bar, uint32_t& phase) {
   const int n = t1 - t0;
   if (threadIdx.x == 0 && n > 0) {
     const uint32_t bytes = static_cast<uint32_t>((n + 3) / 4 * 16);
-    sm100::mbar_arrive_expect_tx(sm100::smem_addr(bar), bytes);
+    sm100::mbar_arrive_expect_tx(sm100::smem_addr(bar), row_u ? 2 * bytes : bytes);
     asm volatile(
         "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(
             sm100::smem_addr(vals)),
         "l"(row + t0), "r"(bytes), "r"(sm100::smem_addr(bar))
         : "memory");
+    if (row_u)
+      asm volatile(
+          "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n" ::"r"(
+              sm100::smem_addr(vals_u)),
+          "l"(row_u + t0), "r"(bytes), "r"(sm100::smem_addr(bar))
+          : "memory");
   }
   bool ok = true;
   if (n > 0) {
     ok = sm100::mbar_wait_bounded(sm100::smem_addr(bar), phase, kWaitLimit);
     phase ^= 1u;
   }
-  if (p.use_T) {
-    for (int i = threadIdx.x; i < n; i += kThreads) vals[i] = __fdiv_rn(vals[i], p.T);
+  if (row_u || p.use_T) {
+    for (int i = threadIdx.x; i < n; i += kThreads) {
+      float x = vals[i];
+      if (row_u) x = adt::cfg_combine(x, vals_u[i], p.cfg);
+      if (p.use_T) x = __fdiv_rn(x, p.T);
+      vals[i] = x;
+    }
   }
   __syncthreads();
   return ok;
@@ -203,7 +218,7 @@ __device__ __forceinline__ float warp_kth_largest(float v, int k, int lane) {
 }
 
 __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) {
-  extern __shared__ __align__(16) float vals[];    // [min(per, kTile)] staged logits
+  extern __shared__ __align__(16) float vals[];    // [min(per, kTile)] staged logits (x2 with guidance)
   __shared__ uint64_t cand[kCandCap];              // keys at or above the CTA's bound
   __shared__ uint64_t wl[kWarps][kMaxK];           // overflow path: each warp's top k
   __shared__ float s_bw[kWarps], s_mw[kWarps], s_sw[kWarps];
@@ -229,6 +244,8 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
   const int c0 = min(p.V, rank * per), c1 = min(p.V, c0 + per);
   const int ntiles = (c1 - c0 + kTile - 1) / kTile;
   const float* row = p.logits + static_cast<int64_t>(r) * p.ld;
+  const float* row_u = p.logits_u ? p.logits_u + static_cast<int64_t>(r) * p.ld : nullptr;
+  float* vals_u = vals + min(per, kTile);  // used only with guidance
 
   for (int i = tid; i < kMaxK; i += kThreads) ctl[i] = 0ull;
   if (tid == 0) {
@@ -246,7 +263,7 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
   for (int tt = 0; tt < ntiles; ++tt) {
     const int t0 = c0 + tt * kTile, t1 = min(c1, t0 + kTile);
     if (tt > 0) __syncthreads();  // the previous tile is consumed
-    ok &= stage_tile(vals, row, t0, t1, p, &s_bar, phase);
+    ok &= stage_tile(vals, vals_u, row, row_u, t0, t1, p, &s_bar, phase);
 #pragma unroll 8
     for (int i = tid; i < t1 - t0; i += kThreads) {
       const float x = vals[i];
@@ -300,7 +317,7 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
     const int t0 = c0 + tt * kTile, t1 = min(c1, t0 + kTile);
     if (ntiles > 1) {
       __syncthreads();
-      ok &= stage_tile(vals, row, t0, t1, p, &s_bar, phase);
+      ok &= stage_tile(vals, vals_u, row, row_u, t0, t1, p, &s_bar, phase);
     }
     const int n = t1 - t0;
     for (int i0 = tid; i0 < n; i0 += 4 * kThreads) {
@@ -337,7 +354,7 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
       const int t0 = c0 + tt * kTile, t1 = min(c1, t0 + kTile);
       if (ntiles > 1) {
         __syncthreads();
-        ok &= stage_tile(vals, row, t0, t1, p, &s_bar, phase);
+        ok &= stage_tile(vals, vals_u, row, row_u, t0, t1, p, &s_bar, phase);
       }
       const int n = t1 - t0;
       for (int base = warp * 32; base < n; base += kThreads) {
@@ -557,21 +574,14 @@ __global__ void __launch_bounds__(kRerankThreads) rerank_kernel(const RerankPara
 
 }  // namespace
 
-extern "C" {
-
-size_t adt_tree_expand_workspace_size(int32_t F, int32_t V, int32_t k_child) {
-  if (F < 1 || V < 1 || k_child < 1) return 0;
-  return expand_ws(F, V, k_child).total;
-}
-
-adt_status adt_tree_expand(const float* logits, int64_t ld, const float* frontier_score,
-                           const int32_t* frontier_id, int32_t F, int32_t V, int32_t k_child,
-                           int32_t k_keep, float temperature, int32_t child_id_base,
-                           int32_t* child_token, float* child_logp, float* child_score,
-                           int32_t* child_parent, int32_t* keep_idx, float* next_score,
-                           int32_t* next_id, void* workspace, size_t workspace_bytes,
-                           void* stream) {
+static adt_status expand_impl(const float* logits, const float* logits_u, float cfg_scale, int64_t ld,
+                              const float* frontier_score, const int32_t* frontier_id, int32_t F, int32_t V,
+                              int32_t k_child, int32_t k_keep, float temperature, int32_t child_id_base,
+                              int32_t* child_token, float* child_logp, float* child_score,
+                              int32_t* child_parent, int32_t* keep_idx, float* next_score, int32_t* next_id,
+                              void* workspace, size_t workspace_bytes, void* stream) {
   ADT_REQUIRE(logits && frontier_score && child_token && child_score && child_parent && keep_idx);
+  if (logits_u) ADT_REQUIRE(adt::aligned16(logits_u) && cfg_scale > -1e30f && cfg_scale < 1e30f);
   ADT_REQUIRE(F >= 1 && F <= kMaxRows && V >= 1 && V <= (1 << 24));
   ADT_REQUIRE(k_child >= 1 && k_child <= kMaxK && k_child <= V);
   ADT_REQUIRE(k_keep >= 1 && k_keep <= F * k_child && k_keep <= kMaxKeep);
@@ -585,6 +595,8 @@ adt_status adt_tree_expand(const float* logits, int64_t ld, const float* frontie
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   ExpandParams p;
   p.logits = logits;
+  p.logits_u = logits_u;
+  p.cfg = cfg_scale;
   p.ld = ld;
   p.fscore = frontier_score;
   p.fid = frontier_id;
@@ -607,13 +619,13 @@ adt_status adt_tree_expand(const float* logits, int64_t ld, const float* frontie
   p.err = info.error_word;
   const int C = expand_cluster(V);
   const int per = ((V + C - 1) / C + 3) & ~3;
-  const size_t dyn = static_cast<size_t>(per < kTile ? per : kTile) * sizeof(float);
+  const size_t dyn = static_cast<size_t>(per < kTile ? per : kTile) * sizeof(float) * (logits_u ? 2 : 1);
   static unsigned configured[2] = {0u, 0u};  // bit per device (< 64)
   unsigned& word = configured[(info.device >> 5) & 1];
   const unsigned bit = 1u << (info.device & 31);
   if (!(__atomic_load_n(&word, __ATOMIC_ACQUIRE) & bit)) {
     ADT_CUDA_TRY(cudaFuncSetAttribute(expand_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      static_cast<int>(kTile * sizeof(float))));
+                                      static_cast<int>(2 * kTile * sizeof(float))));
     __atomic_fetch_or(&word, bit, __ATOMIC_ACQ_REL);
   }
   cudaLaunchConfig_t cfg = {};
@@ -630,6 +642,38 @@ adt_status adt_tree_expand(const float* logits, int64_t ld, const float* frontie
   cfg.numAttrs = 1;
   ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, expand_kernel, p));
   return adt::launch_status();
+}
+
+extern "C" {
+
+size_t adt_tree_expand_workspace_size(int32_t F, int32_t V, int32_t k_child) {
+  if (F < 1 || V < 1 || k_child < 1) return 0;
+  return expand_ws(F, V, k_child).total;
+}
+
+adt_status adt_tree_expand(const float* logits, int64_t ld, const float* frontier_score,
+                           const int32_t* frontier_id, int32_t F, int32_t V, int32_t k_child,
+                           int32_t k_keep, float temperature, int32_t child_id_base,
+                           int32_t* child_token, float* child_logp, float* child_score,
+                           int32_t* child_parent, int32_t* keep_idx, float* next_score,
+                           int32_t* next_id, void* workspace, size_t workspace_bytes,
+                           void* stream) {
+  return expand_impl(logits, nullptr, 0.f, ld, frontier_score, frontier_id, F, V, k_child, k_keep, temperature,
+                     child_id_base, child_token, child_logp, child_score, child_parent, keep_idx, next_score,
+                     next_id, workspace, workspace_bytes, stream);
+}
+
+adt_status adt_tree_expand_cfg(const float* logits_cond, const float* logits_uncond, int64_t ld,
+                               float cfg_scale, const float* frontier_score, const int32_t* frontier_id,
+                               int32_t F, int32_t V, int32_t k_child, int32_t k_keep, float temperature,
+                               int32_t child_id_base, int32_t* child_token, float* child_logp,
+                               float* child_score, int32_t* child_parent, int32_t* keep_idx,
+                               float* next_score, int32_t* next_id, void* workspace,
+                               size_t workspace_bytes, void* stream) {
+  ADT_REQUIRE(logits_uncond);
+  return expand_impl(logits_cond, logits_uncond, cfg_scale, ld, frontier_score, frontier_id, F, V, k_child,
+                     k_keep, temperature, child_id_base, child_token, child_logp, child_score, child_parent,
+                     keep_idx, next_score, next_id, workspace, workspace_bytes, stream);
 }
 
 size_t adt_tree_rerank_workspace_size(int32_t C) {

@@ -129,3 +129,18 @@ def test_controller_rejects_bad_input(lib):
         c.update(0, d + 1)
     with pytest.raises(B.AdtError):
         c.next(16)
+
+
+def test_guidance_entry_points_check_their_extra_arguments(lib):
+    f = ctypes.c_void_p(16)
+    ws = ctypes.c_void_p(256)
+    # expand: no unconditional rows / non-finite scale
+    assert lib.adt_tree_expand_cfg(f, None, 100, 3.0, f, None, 2, 100, 4, 2, 1.0, 0, f, f, f, f, f, None, None, ws,
+                                   1 << 20, None) == 1
+    assert lib.adt_tree_expand_cfg(f, f, 100, float("inf"), f, None, 2, 100, 4, 2, 1.0, 0, f, f, f, f, f, None, None,
+                                   ws, 1 << 20, None) == 1
+    # accept: no unconditional target; SPEC without unconditional draft
+    assert lib.adt_tree_accept_cfg(f, None, 128, None, None, 0, None, 3.0, f, f, f, 1, 100, 8, None, None, 0, 1.0, f,
+                                   8, f, f, None, 0, None) == 1
+    assert lib.adt_tree_accept_cfg(f, f, 128, f, None, 128, None, 3.0, f, f, f, 1, 100, 8, f, f, 1, 1.0, f, 8, f, f,
+                                   None, 0, None) == 1
