@@ -36,6 +36,15 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
     if (adt_e_ != cudaSuccess) return ADT_ERR_CUDA; \
   } while (0)
 
+// Launch attribute that allows a kernel to overlap the tail of the previous
+// one (its device code calls pdl_wait_then_release before touching memory).
+inline cudaLaunchAttribute pdl_attribute() {
+  cudaLaunchAttribute a;
+  a.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  a.val.programmaticStreamSerializationAllowed = 1;
+  return a;
+}
+
 inline adt_status launch_status() {
   return cudaGetLastError() == cudaSuccess ? ADT_OK : ADT_ERR_CUDA;
 }
@@ -43,6 +52,15 @@ inline adt_status launch_status() {
 // ---------------------------------------------------------------- device side
 
 constexpr unsigned kFullMask = 0xffffffffu;
+
+// Programmatic dependent launch: wait until the previous kernel in the
+// stream has completed and its memory is visible (immediate when this launch
+// does not overlap one), then let the next kernel begin launching.  Called
+// before the kernel's first global-memory access.
+__device__ __forceinline__ void pdl_wait_then_release() {
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+}
 
 __device__ __forceinline__ void raise_error(unsigned* word, unsigned bits) {
   if (word) atomicOr(word, bits);

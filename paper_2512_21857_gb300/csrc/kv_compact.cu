@@ -30,6 +30,7 @@ struct CompactParams {
 
 __global__ void __launch_bounds__(kThreads) kv_compact_kernel(const CompactParams p) {
   __shared__ int s_ok;
+  adt::pdl_wait_then_release();
   const int i = blockIdx.x, b = blockIdx.y, l = blockIdx.z, tid = threadIdx.x;
   const int a = p.alen[b];
   const int L = p.kv_len[b];
@@ -113,7 +114,14 @@ adt_status adt_kv_compact(adt_bf16* k_cache, adt_bf16* v_cache, const int32_t* k
   p.tls = tree_layer_stride;
   p.err = info.error_word;
   dim3 grid(static_cast<unsigned>(max_path), static_cast<unsigned>(B), static_cast<unsigned>(num_layers));
-  kv_compact_kernel<<<grid, kThreads, 0, adt::as_stream(stream)>>>(p);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.stream = adt::as_stream(stream);
+  cudaLaunchAttribute attr[1] = {adt::pdl_attribute()};
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, kv_compact_kernel, p));
   return adt::launch_status();
 }
 

@@ -250,6 +250,7 @@ __device__ int cluster_sample(Walker& w, const float* buf, int lo, int cnt, doub
 __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) {
   extern __shared__ __align__(16) float dyn[];
   __shared__ Shared sh;
+  adt::pdl_wait_then_release();
   cg::cluster_group cl = cg::this_cluster();
   Walker w{cl, &sh, static_cast<int>(cl.block_rank()), static_cast<int>(cl.num_blocks()), 0};
   const int b = blockIdx.x / w.csize;
@@ -586,13 +587,14 @@ static adt_status accept_impl(const float* target_logits, const float* target_u,
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = adt::as_stream(stream);
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = cs;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1] = adt::pdl_attribute();
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, accept_kernel, p));
   return adt::launch_status();
 }

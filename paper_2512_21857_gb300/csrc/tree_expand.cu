@@ -232,6 +232,7 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
   __shared__ __align__(8) uint64_t s_bar;
   __shared__ int s_last;
   __shared__ double s_lse;
+  adt::pdl_wait_then_release();
   uint64_t* cross_s = cand;  // cross-row keys (reuses the candidate buffer)
   uint64_t* sel = cand;      // radix path [kMaxKeep]
 
@@ -497,6 +498,7 @@ __global__ void __launch_bounds__(kRerankThreads) rerank_kernel(const RerankPara
   __shared__ int s_tile;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int need = p.n_nodes - 1;
+  adt::pdl_wait_then_release();
   if (tid == 0) {
     p.tokens[0] = *p.root;
     p.parents[0] = -1;
@@ -633,13 +635,14 @@ static adt_status expand_impl(const float* logits, const float* logits_u, float 
   cfg.gridDim = dim3(static_cast<unsigned>(C), static_cast<unsigned>(F), 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.stream = adt::as_stream(stream);
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = static_cast<unsigned>(C);
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1] = adt::pdl_attribute();
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, expand_kernel, p));
   return adt::launch_status();
 }
@@ -709,7 +712,14 @@ adt_status adt_tree_rerank(const int32_t* cand_token, const float* cand_score,
   p.node_of = reinterpret_cast<int32_t*>(ws);
   p.cand_of_node = reinterpret_cast<int32_t*>(ws + adt::align_up(static_cast<size_t>(C) * sizeof(int32_t), 256));
   p.err = info.error_word;
-  rerank_kernel<<<1, kRerankThreads, 0, adt::as_stream(stream)>>>(p);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(1, 1, 1);
+  cfg.blockDim = dim3(kRerankThreads, 1, 1);
+  cfg.stream = adt::as_stream(stream);
+  cudaLaunchAttribute attr[1] = {adt::pdl_attribute()};
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, rerank_kernel, p));
   return adt::launch_status();
 }
 
