@@ -15,7 +15,8 @@
 //   warp 4    TMA tensor loads of prefix K (64 x 64 boxes, 128-byte swizzle)
 //             into a ring of 128-key stages;
 //   warp 5    tcgen05.mma S = Q K^T into one of two tensor-memory tiles
-//             (M = 64 queries, N = 128 keys); frees the K tile once S is done;
+//             (M = 64 queries, N = 128 keys), back to back (softmax warp 0
+//             frees each K tile once it sees its S product done);
 //   warp 6    TMA loads of prefix V into the same stages;
 //   warp 7    tcgen05.mma O += P V (N = head_dim, V read MN-major);
 //   warps 0-3 softmax: warp w owns query rows 16w .. 16w+15 (tensor-memory
@@ -491,9 +492,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           sm100::mma_bf16_ss(tmem + sb * kSCols, da, db, idesc, kk > 0 ? 1u : 0u);
         }
         sm100::mma_commit(sm100::smem_addr(&bars.s_full[sb]));
-        // Once S is done its K tile can be refilled.
-        if (!wait_bar(&bars.s_full[sb], (j >> 1) & 1, &s_abort, p.err)) break;
-        sm100::mbar_arrive(sm100::smem_addr(&bars.k_free[st]));
       }
       if (s_abort) {
         // wait for the tensor core to finish whatever was issued
@@ -552,6 +550,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int j = 0; j < nch; ++j) {
       const int sb = j & 1;
       if (!__all_sync(adt::kFullMask, wait_bar(&bars.s_full[sb], (j >> 1) & 1, &s_abort, p.err))) break;
+      // S(j) is complete, so its K tile can be refilled (the S issuer goes
+      // straight on to the next S product).
+      if (warp == 0 && lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.k_free[j % NS]));
       sm100::tc_fence_after();
       const int keys = chunk_keys(j);
       uint32_t r0[32], r1[32];
