@@ -490,6 +490,87 @@ struct RerankParams {
   unsigned* err;
 };
 
+// Shared-memory rerank for up to kRerankSmall candidates and nodes: a
+// candidate is selected when fewer than n_nodes - 1 candidate keys exceed
+// its own (a warp takes a key and its lanes count), node ids follow
+// ascending candidate index (block scan of the selection flags), and the
+// node maps, parents and depths never leave shared memory.
+constexpr int kRerankSmall = 1024;
+
+__global__ void __launch_bounds__(kRerankThreads) rerank_small_kernel(const RerankParams p) {
+  __shared__ uint64_t keys[kRerankSmall];
+  __shared__ int node_of[kRerankSmall];
+  __shared__ int cand_of_node[kRerankSmall + 1];
+  __shared__ int par[kRerankSmall + 1];
+  __shared__ int warp_tot[32];
+  __shared__ int s_bad;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int need = p.n_nodes - 1, C = p.C;
+  adt::pdl_wait_then_release();
+  if (tid == 0) {
+    p.tokens[0] = *p.root;
+    p.parents[0] = -1;
+    if (p.cand_index) p.cand_index[0] = -1;
+    if (p.depth) p.depth[0] = 0;
+    par[0] = -1;
+    s_bad = 0;
+  }
+  if (need == 0) return;
+  for (int i = tid; i < C; i += kRerankThreads) keys[i] = adt::select_key(p.cscore[i], static_cast<uint32_t>(i));
+  __syncthreads();
+  // selection flag of candidate i (one per thread: C <= kRerankThreads)
+  bool sel = false;
+  for (int i = warp; i < C; i += kRerankThreads / 32) {
+    const uint64_t key = keys[i];
+    int rk = 0;
+    for (int j = 0; j < C; j += 32) rk += __popc(__ballot_sync(adt::kFullMask, j + lane < C && keys[j + lane] > key));
+    if (lane == 0) node_of[i] = rk < need ? 1 : 0;
+  }
+  __syncthreads();
+  if (tid < C) sel = node_of[tid] != 0;
+  // node id = 1 + selected candidates of lower index (block exclusive scan)
+  const unsigned bal = __ballot_sync(adt::kFullMask, sel);
+  if (lane == 0) warp_tot[warp] = __popc(bal);
+  __syncthreads();
+  int before = __popc(bal & ((1u << lane) - 1u));
+  for (int w = 0; w < warp; ++w) before += warp_tot[w];
+  if (tid < C) {
+    const int node = sel ? 1 + before : -1;
+    node_of[tid] = node;
+    if (sel) {
+      cand_of_node[node] = tid;
+      p.tokens[node] = p.ctok[tid];
+      if (p.cand_index) p.cand_index[node] = tid;
+    }
+  }
+  __syncthreads();
+  for (int node = 1 + tid; node <= need; node += kRerankThreads) {
+    const int pc = p.cpar[cand_of_node[node]];
+    int pr = 0;
+    if (pc >= 0) {
+      pr = pc < C ? node_of[pc] : -1;
+      if (pr < 0 || pr >= node) {
+        s_bad = 1;
+        pr = 0;
+      }
+    }
+    par[node] = pr;
+    p.parents[node] = pr;
+  }
+  __syncthreads();
+  if (s_bad && tid == 0) adt::raise_error(p.err, ADT_DEVERR_BAD_TREE);
+  if (p.depth) {
+    for (int node = 1 + tid; node <= need; node += kRerankThreads) {
+      int d = 0, j = node;
+      while (j > 0 && d <= need) {
+        j = par[j];
+        ++d;
+      }
+      p.depth[node] = d;
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kRerankThreads) rerank_kernel(const RerankParams p) {
   __shared__ adt::RadixScratch rs;
   __shared__ int warp_tot[32];
@@ -719,7 +800,10 @@ adt_status adt_tree_rerank(const int32_t* cand_token, const float* cand_score,
   cudaLaunchAttribute attr[1] = {adt::pdl_attribute()};
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, rerank_kernel, p));
+  if (C <= kRerankSmall && C <= kRerankThreads && n_nodes <= kRerankSmall + 1)
+    ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, rerank_small_kernel, p));
+  else
+    ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, rerank_kernel, p));
   return adt::launch_status();
 }
 
