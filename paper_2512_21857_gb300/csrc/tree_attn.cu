@@ -748,23 +748,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     // This owner has its rows, so the copies it was sent are complete.
     sm100::cluster_arrive_relaxed();
     // Thread (row i, column group c4) combines the S partials of that row:
-    // weights 2^(m_c - M) l_c / sum, every split's values loaded up front.
+    // weights 2^(m_c - M) l_c / sum.  A thread takes two items per pass and
+    // loads every split's values of both before combining either.
     // A split without keys sent zeros with m = -inf (weight 0).
-    for (int idx = tid; idx < rows_mine * kC4; idx += kThreads) {
+    auto merge_item = [&](int idx, float2 (&ml)[kMaxClusterSplits], float4 (&v)[kMaxClusterSplits]) {
       const int i = idx / kC4, c4 = idx % kC4;
-      float2 ml[kMaxClusterSplits];
-      float4 v[kMaxClusterSplits];
-#pragma unroll
-      for (int c = 0; c < kMaxClusterSplits; ++c) {
-        if (c < S) {
-          const float* row = slots + (c * rows_per + i) * RS;
-          ml[c] = *reinterpret_cast<const float2*>(row + D);
-          v[c] = *reinterpret_cast<const float4*>(row + c4 * 4);
-        } else {
-          ml[c] = make_float2(-INFINITY, 0.f);
-          v[c] = make_float4(0.f, 0.f, 0.f, 0.f);
-        }
-      }
       float M = ml[0].x;
 #pragma unroll
       for (int c = 1; c < kMaxClusterSplits; ++c) M = fmaxf(M, ml[c].x);
@@ -786,6 +774,29 @@ __global__ void __launch_bounds__(kThreads, 1)
       pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
       *reinterpret_cast<uint2*>(dst) = pk;
       if (c4 == 0 && p.lse) p.lse[static_cast<int64_t>(node0 + r_lo + i) * p.H + h] = (M + log2f(lt)) * kLn2;
+    };
+    auto load_item = [&](int idx, float2 (&ml)[kMaxClusterSplits], float4 (&v)[kMaxClusterSplits]) {
+      const int i = idx / kC4, c4 = idx % kC4;
+#pragma unroll
+      for (int c = 0; c < kMaxClusterSplits; ++c) {
+        if (c < S) {
+          const float* row = slots + (c * rows_per + i) * RS;
+          ml[c] = *reinterpret_cast<const float2*>(row + D);
+          v[c] = *reinterpret_cast<const float4*>(row + c4 * 4);
+        } else {
+          ml[c] = make_float2(-INFINITY, 0.f);
+          v[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      }
+    };
+    for (int idx = tid; idx < rows_mine * kC4; idx += 2 * kThreads) {
+      float2 ml0[kMaxClusterSplits], ml1[kMaxClusterSplits];
+      float4 v0[kMaxClusterSplits], v1[kMaxClusterSplits];
+      const bool two = idx + kThreads < rows_mine * kC4;
+      load_item(idx, ml0, v0);
+      if (two) load_item(idx + kThreads, ml1, v1);
+      merge_item(idx, ml0, v0);
+      if (two) merge_item(idx + kThreads, ml1, v1);
     }
     // Every owner has its rows: this CTA's outgoing copies are complete.
     sm100::cluster_wait_acquire();
