@@ -767,13 +767,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         acc.z += w * v[c].z;
         acc.w += w * v[c].w;
       }
-      const float inv = 1.f / lt;
+      const float inv = __fdividef(1.f, lt);
       __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + r_lo + i) * p.H + h) * D + c4 * 4;
       uint2 pk;
       pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
       pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
       *reinterpret_cast<uint2*>(dst) = pk;
-      if (c4 == 0 && p.lse) p.lse[static_cast<int64_t>(node0 + r_lo + i) * p.H + h] = (M + log2f(lt)) * kLn2;
+      if (c4 == 0 && p.lse) p.lse[static_cast<int64_t>(node0 + r_lo + i) * p.H + h] = (M + __log2f(lt)) * kLn2;
     };
     auto load_item = [&](int idx, float2 (&ml)[kMaxClusterSplits], float4 (&v)[kMaxClusterSplits]) {
       const int i = idx / kC4, c4 = idx % kC4;
