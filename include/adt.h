@@ -121,8 +121,9 @@ const char* adt_status_string(adt_status s);
  * kv_len  [device] int32 [B], prefix length of each tree, 0 <= kv_len <= max_kv.
  * k_tree, v_tree [device] bf16 [Ntot][Hkv][D].
  * parents [device] int32 [Ntot]; node_offsets [device] int32 [B+1].
- * B >= 1; H % Hkv == 0; D in {64, 128}; 1 <= max_nodes <= 64 with every
- *         tree no larger than max_nodes; max_kv >= every kv_len[b].
+ * B >= 1; H % Hkv == 0; D in {64, 128}; 1 <= max_nodes <= 256 with every
+ *         tree no larger than max_nodes (larger trees are processed in
+ *         query tiles of 64 nodes); max_kv >= every kv_len[b].
  * out     [device] bf16 [Ntot][H][D]; lse [device] fp32 [Ntot][H] or NULL.
  * All device pointers 16-byte aligned.  q/out must not alias the caches.
  * Nodes with a malformed tree set ADT_DEVERR_BAD_TREE and their rows are

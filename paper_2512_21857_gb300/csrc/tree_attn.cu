@@ -3,13 +3,15 @@
 // conditioned on s_{1:t} and ans(t) under the tree mask; the mask is the
 // T_N term of Eq. 5).
 //
-// Split-KV flash decoding on the 5th-generation tensor cores.  The keys a
-// tree sees are cut into units of 64: ceil(L/64) prefix units plus one tree
-// unit (its <= 64 nodes, masked per query row by an ancestor bitmask built
-// from the parent pointers).  Grid = (splits, H, B), one CTA per SM; a CTA
-// handles one (tree, head) and a contiguous share of the units, which it
-// walks in chunks: the tree unit first (its K/V are loaded with Q), then the
-// prefix units two at a time (128 keys).
+// Split-KV flash decoding on the 5th-generation tensor cores.  A tree's
+// nodes (<= 256) are cut into query tiles of 64 rows; the keys a tile sees
+// are cut into units of 64: ceil(L/64) prefix units plus the tree units up
+// to its own (a node's ancestors come before it), masked per query row by an
+// ancestor bitmask, one 64-bit word per tree unit, built from the parent
+// pointers.  Grid = (splits, H, B x tiles), one CTA per SM; a CTA handles one
+// (tree, head, tile) and a contiguous share of the units, which it walks in
+// chunks of two units (128 keys): its tree chunks first (their K/V are
+// loaded with Q), then its prefix chunks.
 //
 // Warp roles inside a CTA (256 threads; one thread of each of warps 4-7):
 //   warp 4    TMA tensor loads of prefix K (64 x 64 boxes, 128-byte swizzle)
@@ -48,7 +50,10 @@ namespace {
 
 constexpr int kUnit = 64;               // keys per split unit; the tree unit
 constexpr int kChunk = 128;             // keys per pipeline chunk
-constexpr int kMaxNodes = 64;           // tree nodes (query rows) per (tree, head)
+constexpr int kMaxNodes = 64;           // query rows per CTA: one tile of a tree's nodes
+constexpr int kMaxTreeNodes = 256;      // nodes per tree: up to four query tiles
+constexpr int kMaxTreeUnits = kMaxTreeNodes / kUnit;
+static_assert(kMaxTreeUnits == 4, "the ancestor walk keeps four mask words");
 constexpr int kSoftmaxWarps = 4;
 constexpr int kKLoadWarp = 4;
 constexpr int kSMmaWarp = 5;
@@ -59,9 +64,10 @@ constexpr int kMaxClusterSplits = 8;    // portable cluster size
 constexpr int kMaxSplits = 96;          // workspace merge: weights fit in shared memory
 constexpr int kMaxStages = 4;
 constexpr uint32_t kWaitLimit = 1u << 20;
-constexpr uint32_t kTmemCols = 512;     // two S tiles of 128 columns, then O (<= 128 columns)
+constexpr uint32_t kTmemCols = 512;     // two S tiles of 128 columns, O (<= 128 columns), row sums
 constexpr uint32_t kSCols = 128;
 constexpr uint32_t kOCol = 256;
+constexpr uint32_t kLCols = 16;         // P times a tile of ones: every column holds the row sum
 constexpr float kLn2 = 0.69314718055994530942f;
 constexpr float kLog2e = 1.44269504088896340736f;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
@@ -82,10 +88,15 @@ struct Cfg {
   static constexpr int kStageOff = kPOff + 2 * kPBytes;  // the tree unit's K/V go to slot 0
   static constexpr int kSlotOff = kStageOff + kStages * kStageBytes;  // incoming rows of the merge
   static constexpr int kSlotBytes = (kMaxNodes + kMaxClusterSplits) * kRowStride * 4;
-  static constexpr int kDynSmem = kSlotOff + kSlotBytes + 1024;  // + alignment slack
+  static constexpr int kOnesOff = (kSlotOff + kSlotBytes + 1023) / 1024 * 1024;  // 16 rows of ones (bf16)
+  static constexpr int kOnesBytes = 16 * 128;
+  static constexpr int kDynSmem = kOnesOff + kOnesBytes + 1024;  // + alignment slack
+  static constexpr uint32_t kLCol = kOCol + D;
   static constexpr uint32_t kIdescS128 = sm100::idesc_bf16_f32(64, 128, 0, 0);
   static constexpr uint32_t kIdescS64 = sm100::idesc_bf16_f32(64, 64, 0, 0);
   static constexpr uint32_t kIdescO = sm100::idesc_bf16_f32(64, D, 0, 1);
+  static constexpr uint32_t kIdescL = sm100::idesc_bf16_f32(64, kLCols, 0, 1);
+  static_assert(kLCol + kLCols <= kTmemCols, "tensor memory");
   static_assert(kStages <= kMaxStages, "stage ring");
 };
 
@@ -97,6 +108,7 @@ struct TcParams {
   const int32_t* parents;
   const int32_t* offs;
   int B, H, Hkv, group, max_kv, splits;
+  int qtiles;         // 64-row query tiles per tree: ceil(max_nodes / 64)
   int cluster_merge;
   float scale_log2;
   __nv_bfloat16* out;
@@ -173,6 +185,19 @@ __device__ __forceinline__ void tmem_st_16x256b_x8(uint32_t taddr, const uint32_
       : "memory");
 }
 
+// The same shape, one 8-column block: r[0, 1] row 16w + g, r[2, 3] row 16w + g + 8.
+__device__ __forceinline__ void tmem_ld_16x256b_x1(uint32_t taddr, uint32_t (&r)[4]) {
+  asm volatile("tcgen05.ld.sync.aligned.16x256b.x1.b32 {%0,%1,%2,%3}, [%4];\n"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(taddr)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_st_16x256b_x1(uint32_t taddr, const uint32_t (&r)[4]) {
+  asm volatile("tcgen05.st.sync.aligned.16x256b.x1.b32 [%0], {%1,%2,%3,%4};\n" ::"r"(taddr), "r"(r[0]), "r"(r[1]),
+               "r"(r[2]), "r"(r[3])
+               : "memory");
+}
+
 // x masked to -inf where the keep bit is 0, without branching (a NaN score
 // at a masked position also becomes -inf).
 __device__ __forceinline__ float mask_or_neg_inf(float x, uint32_t keep_bit) {
@@ -183,12 +208,13 @@ __device__ __forceinline__ float mask_or_neg_inf(float x, uint32_t keep_bit) {
 // Softmax of one chunk for the two rows (a, b) a thread holds: NB 8-column
 // blocks (8 for 64 keys, 16 for 128), scores in sa / sb (raw Q.K), keep
 // masks (bit c = column c) applied only when `masked`.  Updates the lazily
-// raised maxima mu (log2 units), the row-sum shares l, returns the rescale
-// factors of O and the bf16 probabilities packed in column pairs.
+// raised maxima mu (log2 units), returns the rescale factors of O (and of
+// the row sums, which the tensor core accumulates from the same bf16
+// probabilities) and the probabilities packed in column pairs.
 template <int NB>
 __device__ __forceinline__ void chunk_softmax(float (&sa)[32], float (&sb)[32], bool masked, uint64_t ka0,
                                               uint64_t ka1, uint64_t kb0, uint64_t kb1, int t4, float scale,
-                                              float& mu_a, float& mu_b, float& l_a, float& l_b, float& alpha_a,
+                                              float& mu_a, float& mu_b, float& alpha_a,
                                               float& alpha_b, uint32_t (&pa)[16], uint32_t (&pb)[16]) {
   if (masked) {
     const int sh = 2 * t4;
@@ -221,20 +247,11 @@ __device__ __forceinline__ void chunk_softmax(float (&sa)[32], float (&sb)[32], 
   alpha_a = needa ? ex2_approx(mu_a - nma) : 1.f;
   alpha_b = needb ? ex2_approx(mu_b - nmb) : 1.f;
   const float base_a = nma == -INFINITY ? 0.f : nma, base_b = nmb == -INFINITY ? 0.f : nmb;
-  float ra[4] = {0.f, 0.f, 0.f, 0.f}, rb[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
   for (int bk = 0; bk < NB; ++bk) {
-    const float a0 = ex2_approx(fmaf(sa[2 * bk], scale, -base_a));
-    const float a1 = ex2_approx(fmaf(sa[2 * bk + 1], scale, -base_a));
-    const float b0 = ex2_approx(fmaf(sb[2 * bk], scale, -base_b));
-    const float b1 = ex2_approx(fmaf(sb[2 * bk + 1], scale, -base_b));
-    ra[bk & 3] += a0 + a1;
-    rb[bk & 3] += b0 + b1;
-    pa[bk] = pack_bf16x2(a0, a1);
-    pb[bk] = pack_bf16x2(b0, b1);
+    pa[bk] = pack_bf16x2(ex2_approx(fmaf(sa[2 * bk], scale, -base_a)), ex2_approx(fmaf(sa[2 * bk + 1], scale, -base_a)));
+    pb[bk] = pack_bf16x2(ex2_approx(fmaf(sb[2 * bk], scale, -base_b)), ex2_approx(fmaf(sb[2 * bk + 1], scale, -base_b)));
   }
-  l_a = l_a * alpha_a + ((ra[0] + ra[1]) + (ra[2] + ra[3]));
-  l_b = l_b * alpha_b + ((rb[0] + rb[1]) + (rb[2] + rb[3]));
   mu_a = nma;
   mu_b = nmb;
 }
@@ -265,7 +282,9 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatil
   return false;
 }
 
-template <int D>
+// kLarge: trees of more than 64 nodes (query tiles, one mask word per tree
+// unit); otherwise one tile and one word, kept in registers.
+template <int D, bool kLarge>
 __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                         const TcParams p) {
@@ -275,14 +294,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   // shared array keeps accesses in the shared address space.
   uint8_t* smem = smem_raw + ((1024u - (sm100::smem_addr(smem_raw) & 1023u)) & 1023u);
   __shared__ Barriers bars;
-  __shared__ uint64_t anc[kMaxNodes];
-  __shared__ int s_par[kMaxNodes];
+  constexpr int kUnits = kLarge ? kMaxTreeUnits : 1;
+  __shared__ uint64_t anc[kMaxNodes][kUnits];
+  __shared__ int s_par[kLarge ? kMaxTreeNodes : kMaxNodes];
   __shared__ uint32_t tmem_slot;
   __shared__ int s_bad;
   __shared__ int s_last;
   __shared__ volatile int s_abort;
 
-  const int split = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int split = blockIdx.x, h = blockIdx.y;
+  const int b = kLarge ? static_cast<int>(blockIdx.z) / p.qtiles : static_cast<int>(blockIdx.z);
+  const int qt = kLarge ? static_cast<int>(blockIdx.z) % p.qtiles : 0;
   const int g = h / p.group;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
@@ -295,34 +317,42 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int total_nodes = p.offs[p.B];
   const int L = p.kv_len[b];
 
-  // Conditions that hold for every CTA of this (tree, head): all leave here.
-  if (n < 1 || n > kMaxNodes || node0 < 0 || node0 + n > total_nodes) {
-    if (split == 0 && h == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_BAD_TREE);
+  // Conditions that hold for every CTA of this (tree, head, tile): all
+  // leave here.  A tile past the end of its tree has no rows.
+  if (n < 1 || n > kMaxNodes * (kLarge ? p.qtiles : 1) || node0 < 0 || node0 + n > total_nodes) {
+    if (split == 0 && h == 0 && qt == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_BAD_TREE);
     return;
   }
   if (L < 0 || L > p.max_kv) {
-    if (split == 0 && h == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_KV_RANGE);
+    if (split == 0 && h == 0 && qt == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_KV_RANGE);
     return;
   }
+  const int row0 = qt * kMaxNodes;  // first node (query row) of this tile
+  const int nq = min(n - row0, kMaxNodes);
+  if (nq <= 0) return;
 
-  // The keys are cut into chunks: ceil(P / 2) prefix chunks of two 64-key
-  // units (P = ceil(L / 64); the last holds one unit when P is odd) and the
-  // tree unit.  Split s takes chunks [s T / S, (s + 1) T / S) of the T; the
-  // split whose share ends with the tree unit processes it first.
+  // The keys are cut into chunks of two 64-key units: ceil(P / 2) prefix
+  // chunks (P = ceil(L / 64); the last holds one unit when P is odd), then
+  // the tree units the tile's rows can see, 0 .. qt (a node's ancestors come
+  // before it), two to a chunk.  Split s takes chunks [s T / S, (s + 1) T / S)
+  // of the T and processes its tree chunks first.
   const int P = (L + kUnit - 1) / kUnit;
-  const int T = (P + 1) / 2 + 1;
+  const int Pc = (P + 1) / 2;
+  const int Tc = kLarge ? (qt + 2) / 2 : 1;  // tree chunks of this tile
+  const int T = Pc + Tc;
   const int S = p.splits;
   const int c_begin = static_cast<int>(static_cast<int64_t>(split) * T / S);
   const int c_end = static_cast<int>(static_cast<int64_t>(split + 1) * T / S);
   const int nch = c_end - c_begin;
-  const int has_tree = (c_end == T && nch > 0) ? 1 : 0;
+  const int tc0 = max(c_begin, Pc) - Pc;         // first tree chunk of this split
+  const int n_tc = max(0, c_end - max(c_begin, Pc));  // its tree chunks, in slots 0 .. n_tc-1
   const int NS = C::kStages;
   auto chunk_keys = [&](int j) -> int {
-    if (has_tree && j == 0) return kUnit;
-    const int pc = c_begin + j - has_tree;
+    if (j < n_tc) return (kLarge && 2 * (tc0 + j) + 1 <= qt ? 2 : 1) * kUnit;
+    const int pc = c_begin + j - n_tc;
     return (2 * pc + 1 < P ? 2 : 1) * kUnit;
   };
-  auto chunk_key0 = [&](int j) -> int { return (c_begin + j - has_tree) * kChunk; };
+  auto chunk_key0 = [&](int j) -> int { return (c_begin + j - n_tc) * kChunk; };
 
   uint8_t* sQ = smem + C::kQOff;
   uint8_t* sP = smem + C::kPOff;
@@ -354,22 +384,36 @@ __global__ void __launch_bounds__(kThreads, 1)
     sm100::tmem_relinquish();
   }
   if (warp < kSoftmaxWarps) {
-    // Q tile: rows node0 .. node0+63 (rows past the tree zero-filled); the
-    // tree unit's K/V for kv head g likewise, into stage slot 0 (the tree is
-    // chunk 0); the parent pointers.
+    // Q tile: rows row0 .. row0+63 of the tree (rows past it zero-filled);
+    // this split's tree chunks (K/V of kv head g, nodes past the tree
+    // zero-filled) into stage slots 0 .. n_tc-1; the parent pointers.
     for (int i = tid; i < kUnit * (D / 8); i += kSoftmaxWarps * 32) {
       const int r = i / (D / 8), ch = i % (D / 8);
-      const bool valid = r < n;
-      const int row = node0 + (valid ? r : 0);
+      const bool valid = r < nq;
+      const int row = node0 + row0 + (valid ? r : 0);
       cp_async16(sm100::smem_addr(sQ) + sw128_off(r, ch, kUnit),
                  p.q + (static_cast<int64_t>(row) * p.H + h) * D + ch * 8, valid ? 16 : 0);
-      if (has_tree) {
+      if (!kLarge && n_tc) {  // the one tree unit: the same rows
         const int64_t off = (static_cast<int64_t>(row) * p.Hkv + g) * D + ch * 8;
         cp_async16(sm100::smem_addr(sStage) + sw128_off(r, ch, kChunk), p.kt + off, valid ? 16 : 0);
         cp_async16(sm100::smem_addr(sStage + C::kStageTile) + sw128_off(r, ch, kChunk), p.vt + off, valid ? 16 : 0);
       }
     }
-    if (tid < n) cp_async4(sm100::smem_addr(&s_par[tid]), p.parents + node0 + tid);
+    for (int jt = 0; kLarge && jt < n_tc; ++jt) {
+      uint8_t* st = sStage + jt * C::kStageBytes;
+      for (int i = tid; i < chunk_keys(jt) * (D / 8); i += kSoftmaxWarps * 32) {
+        const int r = i / (D / 8), ch = i % (D / 8);
+        const int t = (tc0 + jt) * kChunk + r;  // tree node
+        const bool valid = t < n;
+        const int64_t off = (static_cast<int64_t>(node0 + (valid ? t : 0)) * p.Hkv + g) * D + ch * 8;
+        cp_async16(sm100::smem_addr(st) + sw128_off(r, ch, kChunk), p.kt + off, valid ? 16 : 0);
+        cp_async16(sm100::smem_addr(st + C::kStageTile) + sw128_off(r, ch, kChunk), p.vt + off, valid ? 16 : 0);
+      }
+    }
+    for (int t = tid; t < n; t += kSoftmaxWarps * 32) cp_async4(sm100::smem_addr(&s_par[t]), p.parents + node0 + t);
+    // The ones tile (bf16 1.0) of the row-sum product.
+    static_assert(C::kOnesBytes == kSoftmaxWarps * 32 * 16, "one 16-byte store per softmax thread");
+    reinterpret_cast<uint4*>(smem + C::kOnesOff)[tid] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
   }
   sm100::tc_fence_before();
   __syncthreads();
@@ -380,7 +424,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   sm100::cluster_arrive_relaxed();
 
   // Stage loads: chunk j goes to slot j % NS, K tile by warp 4 and V tile by
-  // warp 6.  The tree chunk loads nothing (its K/V came with Q) but still
+  // warp 6.  A tree chunk loads nothing (its K/V came with Q) but still
   // completes its slot's phases, so that every slot's phases advance once
   // per chunk.
   const bool is_loader = (warp == kKLoadWarp || warp == kVLoadWarp) && lane == 0;
@@ -388,7 +432,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto issue_tile = [&](int j) {
     const int st = j % NS;
     const uint32_t bar = sm100::smem_addr(load_v ? &bars.v_full[st] : &bars.k_full[st]);
-    if (has_tree && j == 0) {
+    if (j < n_tc) {
       sm100::mbar_arrive(bar);
       return;
     }
@@ -410,10 +454,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp < kSoftmaxWarps) {
     cp_async_wait_all();
     softmax_warps_sync();
-    // Ancestor bitmask of every node: bit j of anc[t] <=> j in ans(t) or j == t.
-    if (tid < kMaxNodes) {
+    // Ancestor bitmask of every row r of the tile (node t = row0 + r), one
+    // 64-bit word per tree unit: bit j of anc[r][u] <=> node 64u + j is in
+    // ans(t) or is t.  Parents precede their children, so the walk visits
+    // decreasing indices; anything else marks the tree malformed.
+    if (!kLarge && tid < kMaxNodes) {
       uint64_t m = 0;
-      if (tid < n) {
+      if (tid < nq) {
         int j = tid;
         int par = s_par[j];
         m = 1ull << j;
@@ -430,7 +477,42 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (bad) s_bad = 1;
       }
-      anc[tid] = m;
+      anc[tid][0] = m;
+    }
+    if (kLarge && tid < kMaxNodes) {
+      uint64_t m0 = 0, m1 = 0, m2 = 0, m3 = 0;
+      auto set_bit = [&](int j) {
+        const uint64_t bit = 1ull << (j & 63);
+        const int u = j >> 6;
+        m0 |= u == 0 ? bit : 0ull;
+        m1 |= u == 1 ? bit : 0ull;
+        m2 |= u == 2 ? bit : 0ull;
+        m3 |= u == 3 ? bit : 0ull;
+      };
+      if (tid < nq) {
+        int j = row0 + tid;
+        int par = s_par[j];
+        set_bit(j);
+        bool bad = (j == 0) != (par < 0);
+        while (!bad && par >= 0) {
+          if (par >= j) {
+            bad = true;
+            break;
+          }
+          set_bit(par);
+          j = par;
+          par = s_par[j];
+          bad = (j == 0) != (par < 0);
+        }
+        if (bad) s_bad = 1;
+      }
+      uint64_t* w = anc[tid];
+      w[0] = m0;
+      if constexpr (kUnits > 1) {
+        w[1] = m1;
+        w[2] = m2;
+        w[3] = m3;
+      }
     }
   }
   __syncthreads();
@@ -504,6 +586,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ O += P V
     if (lane == 0) {
       const uint32_t p_addr = sm100::smem_addr(sP);
+      // Any 16 K-rows of the ones tile are the same: one descriptor serves
+      // every k step.
+      const uint64_t ones_desc = sm100::smem_desc_sw128(sm100::smem_addr(smem + C::kOnesOff), C::kBlock128, 1024);
       for (int i = 0; i < nch; ++i) {
         if (!wait_bar(&bars.p_full[i & 1], (i >> 1) & 1, &s_abort, p.err) ||
             !wait_bar(&bars.v_full[i % NS], (i / NS) & 1, &s_abort, p.err))
@@ -516,6 +601,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint64_t da = sm100::smem_desc_sw128(pb + (kk >> 2) * C::kBlock64 + (kk & 3) * 32, 16, 1024);
           const uint64_t db = sm100::smem_desc_sw128(v_addr + kk * 2048, C::kBlock128, 1024);  // LBO: d blocks
           sm100::mma_bf16_ss(tmem + kOCol, da, db, C::kIdescO, (i > 0 || kk > 0) ? 1u : 0u);
+          // row sums of the same bf16 P: P times a 16-column tile of ones
+          sm100::mma_bf16_ss(tmem + C::kLCol, da, ones_desc, C::kIdescL, (i > 0 || kk > 0) ? 1u : 0u);
         }
         sm100::mma_commit(sm100::smem_addr(&bars.done[i % NS]));
       }
@@ -537,16 +624,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     // of a quad share a row and combine row statistics with two shuffles.
     const int g8 = lane >> 2, t4 = lane & 3;
     const int ra = warp * 16 + g8, rb = ra + 8;
-    const uint64_t ama = ra < n ? anc[ra] : 0ull;
-    const uint64_t amb = rb < n ? anc[rb] : 0ull;
     const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
     // stmatrix addressing: lane l writes row (l / 8 odd ? 8 : 0) + l % 8 of
     // the warp's rows, in column block (l / 16) of each pair of blocks.
     const int st_row = warp * 16 + ((lane >> 3) & 1) * 8 + (lane & 7);
     const int st_blk = lane >> 4;
     const float scale = p.scale_log2;
+    const uint64_t ama = anc[ra][0], amb = anc[rb][0];  // the one tree unit (kLarge: unused)
     float mua = -INFINITY, mub = -INFINITY;  // running maxima used for the exponentials
-    float la = 0.f, lb = 0.f;                // this thread's share of the row sums
     for (int j = 0; j < nch; ++j) {
       const int sb = j & 1;
       if (!__all_sync(adt::kFullMask, wait_bar(&bars.s_full[sb], (j >> 1) & 1, &s_abort, p.err))) break;
@@ -567,13 +652,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       // Which keys a row sees: its ancestors and itself in the tree unit,
       // the prefix up to L otherwise.  Only the tree chunk and a chunk that
       // holds the end of the prefix need a mask.
-      const bool tree_j = has_tree && j == 0;
+      const bool tree_j = j < n_tc;
       const int kl = tree_j ? keys : L - chunk_key0(j);
       const bool masked = tree_j || kl < keys;
       uint64_t ka0 = ~0ull, ka1 = ~0ull, kb0 = ~0ull, kb1 = ~0ull;
       if (tree_j) {
-        ka0 = ama;
-        kb0 = amb;
+        if constexpr (kLarge) {
+          // units 2u and 2u + 1 of the tree (rows past the tile have no bits)
+          const int u = 2 * (tc0 + j);
+          ka0 = anc[ra][u];
+          kb0 = anc[rb][u];
+          ka1 = u + 1 < kUnits ? anc[ra][u + 1] : 0ull;
+          kb1 = u + 1 < kUnits ? anc[rb][u + 1] : 0ull;
+        } else {
+          ka0 = ama;
+          kb0 = amb;
+        }
       } else if (kl < keys) {
         ka0 = kb0 = kl >= 64 ? ~0ull : ((1ull << kl) - 1ull);
         ka1 = kb1 = kl >= 128 ? ~0ull : (kl > 64 ? ((1ull << (kl - 64)) - 1ull) : 0ull);
@@ -593,9 +687,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t pa[16], pb[16];
       float alpha_a, alpha_b;
       if (keys == kChunk)
-        chunk_softmax<16>(sa, sbv, masked, ka0, ka1, kb0, kb1, t4, scale, mua, mub, la, lb, alpha_a, alpha_b, pa, pb);
+        chunk_softmax<16>(sa, sbv, masked, ka0, ka1, kb0, kb1, t4, scale, mua, mub, alpha_a, alpha_b, pa, pb);
       else
-        chunk_softmax<8>(sa, sbv, masked, ka0, ka1, kb0, kb1, t4, scale, mua, mub, la, lb, alpha_a, alpha_b, pa, pb);
+        chunk_softmax<8>(sa, sbv, masked, ka0, ka1, kb0, kb1, t4, scale, mua, mub, alpha_a, alpha_b, pa, pb);
 
       // P buffer sb was last read by the PV product of chunk j - 2.
       if (j >= 2 && !__all_sync(adt::kFullMask,
@@ -646,21 +740,24 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tmem_st_16x256b_x8(tmem + lane_base + kOCol + c0, o);
         }
+        {
+          uint32_t l4[4];
+          tmem_ld_16x256b_x1(tmem + lane_base + C::kLCol, l4);
+          sm100::tmem_wait_ld();
+          l4[0] = __float_as_uint(__uint_as_float(l4[0]) * alpha_a);
+          l4[1] = __float_as_uint(__uint_as_float(l4[1]) * alpha_a);
+          l4[2] = __float_as_uint(__uint_as_float(l4[2]) * alpha_b);
+          l4[3] = __float_as_uint(__uint_as_float(l4[3]) * alpha_b);
+          tmem_st_16x256b_x1(tmem + lane_base + C::kLCol, l4);
+        }
         sm100::tmem_wait_st();
       }
       sm100::tc_fence_before();
       __syncwarp();
       if (lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.p_full[sb]));
     }
-    // Full row sums: add the four shares of each quad.
-    la += __shfl_xor_sync(adt::kFullMask, la, 1);
-    la += __shfl_xor_sync(adt::kFullMask, la, 2);
-    lb += __shfl_xor_sync(adt::kFullMask, lb, 1);
-    lb += __shfl_xor_sync(adt::kFullMask, lb, 2);
     m_ra = mua;
-    l_ra = la;
     m_rb = mub;
-    l_rb = lb;
   }
 
   // ------------------------------------------------------------ epilogue
@@ -680,7 +777,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
 #pragma unroll
       for (int c = 0; c < kOB; ++c) tmem_ld_16x256b_x8(tmem + lane_base + kOCol + c * 64, o[c]);
+      uint32_t l4[4];
+      tmem_ld_16x256b_x1(tmem + lane_base + C::kLCol, l4);  // every column holds the row sum
       sm100::tmem_wait_ld();
+      l_ra = __uint_as_float(l4[0]);
+      l_rb = __uint_as_float(l4[2]);
     } else {
       // A split without key units (kv_len shorter than max_kv) contributes
       // nothing: weight 0.
@@ -692,18 +793,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int g8 = lane >> 2, t4 = lane & 3;
   const int ra = warp * 16 + g8, rb = ra + 8;
-  const int64_t bh = static_cast<int64_t>(b) * p.H + h;
+  const int64_t bh = static_cast<int64_t>(blockIdx.z) * p.H + h;  // (tree, tile, head)
   constexpr int kC4 = D / 4;
   if (p.cluster_merge) {
-    // Row r of the (tree, head) is merged by split r / rows_per, its owner.
+    // Row r of the (tree, head, tile) is merged by split r / rows_per, its owner.
     // Each split writes its partial rows (O unnormalised, then m and l) into
     // its own stage ring, idle now, in row order; one thread sends every
     // owner its rows with bulk shared-to-shared copies into the owner's slot
     // region, completing on the owner's mbarrier; each owner merges locally.
     constexpr int RS = C::kRowStride;
-    const int rows_per = (n + S - 1) / S;
+    const int rows_per = (nq + S - 1) / S;
     const int r_lo = split * rows_per;
-    const int rows_mine = max(0, min(n, r_lo + rows_per) - r_lo);
+    const int rows_mine = max(0, min(nq, r_lo + rows_per) - r_lo);
     float* rows_out = reinterpret_cast<float*>(sStage);
     if (tid == 0)
       sm100::mbar_arrive_expect_tx(sm100::smem_addr(&bars.recv), static_cast<uint32_t>(S * rows_mine * RS * 4));
@@ -711,7 +812,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int half = 0; half < 2; ++half) {
         const int r = half ? rb : ra;
-        if (r < n) {
+        if (r < nq) {
           float* dst = rows_out + r * RS;
           if (t4 == 0) *reinterpret_cast<float2*>(dst + D) = half ? make_float2(m_rb, l_rb) : make_float2(m_ra, l_ra);
 #pragma unroll
@@ -733,7 +834,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     sm100::cluster_wait_acquire();
     if (tid == 0) {
       for (int c = 0; c < S; ++c) {
-        const int rc = max(0, min(n, (c + 1) * rows_per) - c * rows_per);
+        const int rc = max(0, min(nq, (c + 1) * rows_per) - c * rows_per);
         if (rc > 0)
           sm100::bulk_copy_to_cluster(sm100::mapa_shared(sm100::smem_addr(slots + split * rows_per * RS), c),
                                       sm100::smem_addr(rows_out + c * rows_per * RS),
@@ -768,12 +869,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         acc.w += w * v[c].w;
       }
       const float inv = __fdividef(1.f, lt);
-      __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + r_lo + i) * p.H + h) * D + c4 * 4;
+      __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + row0 + r_lo + i) * p.H + h) * D + c4 * 4;
       uint2 pk;
       pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
       pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
       *reinterpret_cast<uint2*>(dst) = pk;
-      if (c4 == 0 && p.lse) p.lse[static_cast<int64_t>(node0 + r_lo + i) * p.H + h] = (M + __log2f(lt)) * kLn2;
+      if (c4 == 0 && p.lse) p.lse[static_cast<int64_t>(node0 + row0 + r_lo + i) * p.H + h] = (M + __log2f(lt)) * kLn2;
     };
     auto load_item = [&](int idx, float2 (&ml)[kMaxClusterSplits], float4 (&v)[kMaxClusterSplits]) {
       const int i = idx / kC4, c4 = idx % kC4;
@@ -813,7 +914,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
       const int r = half ? rb : ra;
-      if (r < n) {
+      if (r < nq) {
         if (t4 == 0) pml[r] = half ? make_float2(m_rb, l_rb) : make_float2(m_ra, l_ra);
 #pragma unroll
         for (int c = 0; c < kOB; ++c) {
@@ -840,7 +941,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const float* po_bh = p.part_o + bh * S * kMaxNodes * D;
   const float2* pml_bh = p.part_ml + bh * S * kMaxNodes;
   float* wsm = reinterpret_cast<float*>(sStage);  // [64][S]
-  if (tid < n) {
+  if (tid < nq) {
     float M = -INFINITY;
     for (int sp = 0; sp < S; ++sp) M = fmaxf(M, __ldcg(&pml_bh[sp * kMaxNodes + tid]).x);
     float lt = 0.f;
@@ -852,11 +953,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     const float inv = 1.f / lt;
     for (int sp = 0; sp < S; ++sp) wsm[tid * S + sp] *= inv;
-    if (p.lse) p.lse[static_cast<int64_t>(node0 + tid) * p.H + h] = (M + log2f(lt)) * kLn2;
+    if (p.lse) p.lse[static_cast<int64_t>(node0 + row0 + tid) * p.H + h] = (M + log2f(lt)) * kLn2;
   }
   __syncthreads();
   constexpr int kStride4 = kMaxNodes * D / 4;
-  for (int idx = tid; idx < n * kC4; idx += kThreads) {
+  for (int idx = tid; idx < nq * kC4; idx += kThreads) {
     const int rr = idx / kC4, c4 = idx % kC4;
     const float4* src = reinterpret_cast<const float4*>(po_bh + rr * D) + c4;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -882,7 +983,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       acc.z += w * v.z;
       acc.w += w * v.w;
     }
-    __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + rr) * p.H + h) * D + c4 * 4;
+    __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + row0 + rr) * p.H + h) * D + c4 * 4;
     uint2 pk;
     pk.x = pack_bf16x2(acc.x, acc.y);
     pk.y = pack_bf16x2(acc.z, acc.w);
@@ -898,17 +999,20 @@ __global__ void __launch_bounds__(kThreads, 1)
 // lowered until all B*H clusters are co-resident (GPC sizes decide how many
 // clusters of a given size fit at once).  Many splits (small B*H, long
 // prefixes) merge through the workspace instead.
-int max_active_clusters(int D, int cluster, int dev);
+int max_active_clusters(int D, bool large, int cluster, int dev);
 
-int choose_splits(int sm_count, int B, int H, int D, int max_kv, int dev) {
+int qtiles_for(int max_nodes) { return (max_nodes + kMaxNodes - 1) / kMaxNodes; }
+
+// Bq = trees x query tiles.
+int choose_splits(int sm_count, int Bq, int H, int D, int max_kv, int dev, bool large) {
   const int units = ((max_kv + kUnit - 1) / kUnit + 1) / 2 + 1;  // chunks, the tree unit included
-  const int bh = B * H;
+  const int bh = Bq * H;
   int s = sm_count / bh;
   if (s < 1) s = 1;
   if (s > units) s = units;
   if (s >= 2 * kMaxClusterSplits) return s > kMaxSplits ? kMaxSplits : s;
   if (s > kMaxClusterSplits) s = kMaxClusterSplits;
-  while (s > 1 && max_active_clusters(D, s, dev) < bh) --s;
+  while (s > 1 && max_active_clusters(D, large, s, dev) < bh) --s;
   return s;
 }
 
@@ -966,9 +1070,21 @@ adt_status make_cache_map(CUtensorMap* map, const void* base, int D, int max_kv,
   return r == CUDA_SUCCESS ? ADT_OK : ADT_ERR_INVALID_ARG;
 }
 
-int max_active_clusters(int D, int cluster, int dev) {
-  static int cache[64][2][kMaxClusterSplits + 1];  // 0 = not queried yet
-  int& slot = cache[dev & 63][D == 128 ? 1 : 0][cluster];
+template <int D, bool kLarge>
+int occupancy_clusters(cudaLaunchConfig_t* cfg) {
+  int num = 0;
+  cudaFuncSetAttribute(tree_attn_tc_kernel<D, kLarge>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<D>::kDynSmem);
+  cfg->dynamicSmemBytes = Cfg<D>::kDynSmem;
+  if (cudaOccupancyMaxActiveClusters(&num, tree_attn_tc_kernel<D, kLarge>, cfg) != cudaSuccess) {
+    (void)cudaGetLastError();
+    num = 0;
+  }
+  return num;
+}
+
+int max_active_clusters(int D, bool large, int cluster, int dev) {
+  static int cache[64][2][2][kMaxClusterSplits + 1];  // 0 = not queried yet
+  int& slot = cache[dev & 63][D == 128 ? 1 : 0][large ? 1 : 0][cluster];
   int v = __atomic_load_n(&slot, __ATOMIC_ACQUIRE);
   if (v) return v - 1;
   cudaLaunchConfig_t cfg = {};
@@ -981,33 +1097,20 @@ int max_active_clusters(int D, int cluster, int dev) {
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  int num = 0;
-  cudaError_t e;
-  if (D == 128) {
-    cudaFuncSetAttribute(tree_attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<128>::kDynSmem);
-    cfg.dynamicSmemBytes = Cfg<128>::kDynSmem;
-    e = cudaOccupancyMaxActiveClusters(&num, tree_attn_tc_kernel<128>, &cfg);
-  } else {
-    cudaFuncSetAttribute(tree_attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<64>::kDynSmem);
-    cfg.dynamicSmemBytes = Cfg<64>::kDynSmem;
-    e = cudaOccupancyMaxActiveClusters(&num, tree_attn_tc_kernel<64>, &cfg);
-  }
-  if (e != cudaSuccess) {
-    (void)cudaGetLastError();
-    num = 0;
-  }
+  const int num = D == 128 ? (large ? occupancy_clusters<128, true>(&cfg) : occupancy_clusters<128, false>(&cfg))
+                           : (large ? occupancy_clusters<64, true>(&cfg) : occupancy_clusters<64, false>(&cfg));
   __atomic_store_n(&slot, num + 1, __ATOMIC_RELEASE);
   return num;
 }
 
-template <int D>
+template <int D, bool kLarge>
 adt_status launch(TcParams prm, const void* k_cache, const void* v_cache, int64_t sb, int64_t sh, cudaStream_t st,
                   int dev, bool overlap_previous) {
-  static unsigned configured[2] = {0u, 0u};  // bit per device (< 64)
+  static unsigned configured[2] = {0u, 0u};  // bit per device (< 64), per instantiation
   const unsigned bit = 1u << (dev & 31);
   unsigned& word = configured[dev >> 5];
   if (!(__atomic_load_n(&word, __ATOMIC_ACQUIRE) & bit)) {
-    ADT_CUDA_TRY(cudaFuncSetAttribute(tree_attn_tc_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    ADT_CUDA_TRY(cudaFuncSetAttribute(tree_attn_tc_kernel<D, kLarge>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                       Cfg<D>::kDynSmem));
     __atomic_fetch_or(&word, bit, __ATOMIC_ACQ_REL);
   }
@@ -1018,7 +1121,8 @@ adt_status launch(TcParams prm, const void* k_cache, const void* v_cache, int64_
   if (s1 != ADT_OK) return s1;
   prm.cluster_merge = prm.splits <= kMaxClusterSplits ? 1 : 0;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(prm.splits), static_cast<unsigned>(prm.H), static_cast<unsigned>(prm.B));
+  cfg.gridDim = dim3(static_cast<unsigned>(prm.splits), static_cast<unsigned>(prm.H),
+                     static_cast<unsigned>(prm.B * prm.qtiles));
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = Cfg<D>::kDynSmem;
   cfg.stream = st;
@@ -1033,8 +1137,19 @@ adt_status launch(TcParams prm, const void* k_cache, const void* v_cache, int64_
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = overlap_previous ? 2 : 1;
-  ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, tree_attn_tc_kernel<D>, tm_k, tm_v, prm));
+  ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, tree_attn_tc_kernel<D, kLarge>, tm_k, tm_v, prm));
   return adt::launch_status();
+}
+
+// Trees of more than 64 nodes take the query-tiled instantiation.
+adt_status launch_any(const TcParams& prm, int D, const void* k_cache, const void* v_cache, int64_t sb, int64_t sh,
+                      cudaStream_t st, int dev, bool overlap_previous) {
+  const bool large = prm.qtiles > 1;
+  if (D == 128)
+    return large ? launch<128, true>(prm, k_cache, v_cache, sb, sh, st, dev, overlap_previous)
+                 : launch<128, false>(prm, k_cache, v_cache, sb, sh, st, dev, overlap_previous);
+  return large ? launch<64, true>(prm, k_cache, v_cache, sb, sh, st, dev, overlap_previous)
+               : launch<64, false>(prm, k_cache, v_cache, sb, sh, st, dev, overlap_previous);
 }
 
 // Shared host checks of both entry points.
@@ -1044,11 +1159,12 @@ adt_status check_args(const adt_bf16* q, const adt_bf16* k_cache, const adt_bf16
                       int32_t D, int32_t max_nodes, int32_t max_kv, float scale, const adt_bf16* out) {
   ADT_REQUIRE(q && k_cache && v_cache && kv_len && k_tree && v_tree && parents && node_offsets && out);
   ADT_REQUIRE(B >= 1 && H >= 1 && Hkv >= 1 && H % Hkv == 0);
-  ADT_REQUIRE(static_cast<int64_t>(B) * H <= kMaxBH && B <= 65535 && H <= 65535);
   ADT_REQUIRE(max_nodes >= 1 && max_kv >= 0 && max_kv < (1 << 30));
+  if (max_nodes > kMaxTreeNodes) return ADT_ERR_UNSUPPORTED;
+  const int64_t bq = static_cast<int64_t>(B) * qtiles_for(max_nodes);
+  ADT_REQUIRE(bq * H <= kMaxBH && bq <= 65535 && H <= 65535);
   ADT_REQUIRE(scale > 0.f && scale < 1e30f);
   if (D != 64 && D != 128) return ADT_ERR_UNSUPPORTED;
-  if (max_nodes > kMaxNodes) return ADT_ERR_UNSUPPORTED;
   ADT_REQUIRE(sb >= 0 && sh >= 0 && sb % 8 == 0 && sh % 8 == 0);
   ADT_REQUIRE(Hkv == 1 || sh >= static_cast<int64_t>(max_kv) * D);
   ADT_REQUIRE(B == 1 || sb >= static_cast<int64_t>(max_kv) * D);
@@ -1059,7 +1175,7 @@ adt_status check_args(const adt_bf16* q, const adt_bf16* k_cache, const adt_bf16
 
 TcParams make_params(const adt_bf16* q, const int32_t* kv_len, const adt_bf16* k_tree, const adt_bf16* v_tree,
                      const int32_t* parents, const int32_t* node_offsets, int B, int H, int Hkv, int max_kv,
-                     int splits, float scale, adt_bf16* out, float* lse, unsigned* err) {
+                     int max_nodes, int splits, float scale, adt_bf16* out, float* lse, unsigned* err) {
   TcParams prm{};
   prm.q = reinterpret_cast<const __nv_bfloat16*>(q);
   prm.kt = reinterpret_cast<const __nv_bfloat16*>(k_tree);
@@ -1073,6 +1189,7 @@ TcParams make_params(const adt_bf16* q, const int32_t* kv_len, const adt_bf16* k
   prm.group = H / Hkv;
   prm.max_kv = max_kv;
   prm.splits = splits;
+  prm.qtiles = qtiles_for(max_nodes);
   prm.scale_log2 = scale * kLog2e;
   prm.out = reinterpret_cast<__nv_bfloat16*>(out);
   prm.lse = lse;
@@ -1086,11 +1203,12 @@ extern "C" {
 
 size_t adt_tree_attn_workspace_size(int32_t B, int32_t H, int32_t D, int32_t max_nodes,
                                     int32_t max_kv) {
-  (void)max_nodes;
-  if (B < 1 || H < 1 || (D != 64 && D != 128) || max_kv < 0 || static_cast<int64_t>(B) * H > kMaxBH) return 0;
+  if (B < 1 || H < 1 || (D != 64 && D != 128) || max_kv < 0 || max_nodes < 1 || max_nodes > kMaxTreeNodes) return 0;
+  const int Bq = B * qtiles_for(max_nodes);
+  if (static_cast<int64_t>(Bq) * H > kMaxBH) return 0;
   adt::DeviceInfo info;
   if (adt::device_info(&info) != ADT_OK) return 0;
-  return ws_layout(B, H, D, choose_splits(info.sm_count, B, H, D, max_kv, info.device)).total;
+  return ws_layout(Bq, H, D, choose_splits(info.sm_count, Bq, H, D, max_kv, info.device, max_nodes > kMaxNodes)).total;
 }
 
 adt_status adt_tree_attn(const adt_bf16* q, const adt_bf16* k_cache, const adt_bf16* v_cache,
@@ -1105,18 +1223,18 @@ adt_status adt_tree_attn(const adt_bf16* q, const adt_bf16* k_cache, const adt_b
   adt::DeviceInfo info;
   st = adt::device_info(&info);
   if (st != ADT_OK) return st;
-  const int splits = choose_splits(info.sm_count, B, H, D, max_kv, info.device);
-  const WsLayout w = ws_layout(B, H, D, splits);
+  const int Bq = B * qtiles_for(max_nodes);
+  const int splits = choose_splits(info.sm_count, Bq, H, D, max_kv, info.device, max_nodes > kMaxNodes);
+  const WsLayout w = ws_layout(Bq, H, D, splits);
   if (!workspace || workspace_bytes < w.total || !adt::aligned16(workspace)) return ADT_ERR_WORKSPACE;
   uint8_t* ws = static_cast<uint8_t*>(workspace);
-  TcParams prm = make_params(q, kv_len, k_tree, v_tree, parents, node_offsets, B, H, Hkv, max_kv, splits,
+  TcParams prm = make_params(q, kv_len, k_tree, v_tree, parents, node_offsets, B, H, Hkv, max_kv, max_nodes, splits,
                              softmax_scale, out, lse, info.error_word);
   prm.part_o = reinterpret_cast<float*>(ws + w.part_o);
   prm.part_ml = reinterpret_cast<float2*>(ws + w.part_ml);
   prm.tickets = reinterpret_cast<unsigned*>(ws + w.tickets);
   cudaStream_t s = adt::as_stream(stream);
-  return D == 128 ? launch<128>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device, true)
-                  : launch<64>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device, true);
+  return launch_any(prm, D, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device, true);
 }
 
 }  // extern "C"
@@ -1188,19 +1306,19 @@ extern "C" adt_status adt_tree_attn_noalloc(const adt_bf16* q, const adt_bf16* k
   if (g_noalloc_status[info.device] != cudaSuccess || !g_noalloc_ptr[info.device]) return ADT_ERR_CUDA;
   // As many splits as the usual heuristic picks, fewer if the partials would
   // not fit; a shape that does not fit even unsplit is rejected.
-  int splits = choose_splits(info.sm_count, B, H, D, max_kv, info.device);
-  while (splits > 1 && noalloc_layout(B, H, D, splits).total > kNoAllocScratchBytes) --splits;
-  const NoAllocLayout w = noalloc_layout(B, H, D, splits);
+  const int Bq = B * qtiles_for(max_nodes);
+  int splits = choose_splits(info.sm_count, Bq, H, D, max_kv, info.device, max_nodes > kMaxNodes);
+  while (splits > 1 && noalloc_layout(Bq, H, D, splits).total > kNoAllocScratchBytes) --splits;
+  const NoAllocLayout w = noalloc_layout(Bq, H, D, splits);
   if (w.total > kNoAllocScratchBytes) return ADT_ERR_WORKSPACE;
   uint8_t* ws = static_cast<uint8_t*>(g_noalloc_ptr[info.device]);
   cudaStream_t s = adt::as_stream(stream);
   // The array keeps the previous call's contents: the tickets must start at zero.
-  ADT_CUDA_TRY(cudaMemsetAsync(ws + w.tickets, 0, static_cast<size_t>(B) * H * sizeof(unsigned), s));
-  TcParams prm = make_params(q, kv_len, k_tree, v_tree, parents, node_offsets, B, H, Hkv, max_kv, splits,
+  ADT_CUDA_TRY(cudaMemsetAsync(ws + w.tickets, 0, static_cast<size_t>(Bq) * H * sizeof(unsigned), s));
+  TcParams prm = make_params(q, kv_len, k_tree, v_tree, parents, node_offsets, B, H, Hkv, max_kv, max_nodes, splits,
                              softmax_scale, out, lse, info.error_word);
   prm.part_o = reinterpret_cast<float*>(ws + w.part_o);
   prm.part_ml = reinterpret_cast<float2*>(ws + w.part_ml);
   prm.tickets = reinterpret_cast<unsigned*>(ws + w.tickets);
-  return D == 128 ? launch<128>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device, false)
-                  : launch<64>(prm, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device, false);
+  return launch_any(prm, D, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device, false);
 }

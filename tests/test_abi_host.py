@@ -52,8 +52,8 @@ def test_invalid_arguments_rejected_before_launch(lib):
     assert lib.adt_tree_attn(None, f, f, f, 0, 0, f, f, f, f, 1, 1, 1, 64, 1, 1, 1.0, f, None, f, 0, None) == 1
     # head_dim outside {64, 128} -> unsupported
     assert lib.adt_tree_attn(f, f, f, f, 0, 0, f, f, f, f, 1, 1, 1, 96, 1, 1, 1.0, f, None, f, 0, None) == 2
-    # more than 64 nodes per tree -> unsupported
-    assert lib.adt_tree_attn(f, f, f, f, 0, 0, f, f, f, f, 1, 1, 1, 64, 65, 1, 1.0, f, None, f, 0, None) == 2
+    # more than 256 nodes per tree -> unsupported
+    assert lib.adt_tree_attn(f, f, f, f, 0, 0, f, f, f, f, 1, 1, 1, 64, 257, 1, 1.0, f, None, f, 0, None) == 2
     # H not a multiple of Hkv
     assert lib.adt_tree_attn(f, f, f, f, 0, 0, f, f, f, f, 1, 3, 2, 64, 8, 1, 1.0, f, None, f, 0, None) == 1
     # expand: k_child > 64, k_keep > F*k, ld not a multiple of 4

@@ -4,7 +4,7 @@
 import numpy as np
 import pytest
 
-from gpu_cases import AttnCase, assert_attention_close, ensure_built
+from gpu_cases import LSE_ATOL, AttnCase, assert_attention_close, ensure_built
 
 pytestmark = pytest.mark.gpu
 
@@ -31,7 +31,38 @@ def test_attention_matches_oracle(sizes, kv, H, Hkv, D):
     got, lse, _ = case.run_gpu()
     ref, ref_lse = case.run_oracle()
     assert_attention_close(got, ref)
-    assert np.abs(lse - ref_lse).max() < 2e-3
+    assert np.abs(lse - ref_lse).max() < LSE_ATOL
+
+
+# Trees of more than 64 nodes (width bound 39 for LlamaGen-class drafts):
+# 64-row query tiles, each seeing the tree units up to its own.
+LARGE_CASES = [
+    # sizes, kv_lens, H, Hkv, D
+    ([256], [600], 8, 8, 128),                  # four full query tiles
+    ([100], [2400], 16, 16, 128),               # second tile partial, long prefix
+    ([65], [0], 4, 4, 64),                      # one node in the second tile, empty prefix
+    ([200, 7, 129], [700, 64, 1], 8, 2, 128),   # ragged batch across tile counts, grouped kv heads
+    ([192], [696], 20, 20, 64),                 # LlamaGen-XL-shaped layer, three tiles
+]
+
+
+@pytest.mark.parametrize("sizes,kv,H,Hkv,D", LARGE_CASES)
+def test_large_tree_matches_oracle(sizes, kv, H, Hkv, D):
+    case = AttnCase(sizes, kv, H, Hkv, D, seed=301 + sum(sizes), max_depth=10, max_children=39)
+    got, lse, _ = case.run_gpu(max_nodes=max(sizes))
+    ref, ref_lse = case.run_oracle()
+    assert_attention_close(got, ref)
+    assert np.abs(lse - ref_lse).max() < LSE_ATOL
+
+
+@pytest.mark.parametrize("chain", [True, False])
+def test_256_node_extremes(chain):
+    """A 256-node chain (every mask word full below the diagonal) and a
+    256-node star (each node sees the root and itself)."""
+    case = AttnCase([256], [130], 4, 4, 128, seed=9, chain=chain, max_depth=1, max_children=255)
+    got, _, _ = case.run_gpu(max_nodes=256)
+    ref, _ = case.run_oracle()
+    assert_attention_close(got, ref)
 
 
 def test_chain_tree_matches_oracle():
@@ -48,7 +79,7 @@ def test_7b_shape_one_layer_full_size():
     got, lse, _ = case.run_gpu(max_kv=2400 + 64)
     ref, ref_lse = case.run_oracle()
     assert_attention_close(got, ref)
-    assert np.abs(lse - ref_lse).max() < 2e-3
+    assert np.abs(lse - ref_lse).max() < LSE_ATOL
 
 
 def test_batch_of_eight_ragged_prefixes():
