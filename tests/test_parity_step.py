@@ -90,3 +90,16 @@ def test_step_llamagen_shape():
     step.launch()
     torch.cuda.synchronize()
     assert _check(step, inp, tree, B.ACCEPT_GREEDY, layers=[0, 1]) >= 2
+
+
+@pytest.mark.parametrize("mode,plant", [(B.ACCEPT_GREEDY, 3), (B.ACCEPT_SPEC_DET, 0)])
+def test_step_llamagen_width_39_tree_of_256(mode, plant):
+    """LlamaGen-class width bound (k = 39, Sec. 5.1): 39 + 4 * 39^2
+    candidates, the 255 best kept, so attention runs four query tiles."""
+    step, inp, tree = _setup(2, 20, 64, 16384, 696, 5, 39, 256, mode, seed=12 + mode, plant=plant)
+    assert len(tree["tokens"]) == 256
+    step.launch()
+    torch.cuda.synchronize()
+    a = _check(step, inp, tree, mode, layers=[0, 1])
+    if mode == B.ACCEPT_GREEDY:
+        assert a >= 2
