@@ -340,6 +340,31 @@ adt_status adt_kv_compact(adt_bf16* k_cache, adt_bf16* v_cache, const int32_t* k
                           int64_t tree_layer_stride, void* stream);
 
 /* ------------------------------------------------------------------------
+ * adt_kv_compact_inplace - adt_kv_compact for a cache that already holds
+ * the tree's K/V in its tail (the tree written right after the prefix, as
+ * engines that append draft tokens to the cache do): row kv_len[b] + t of
+ * tree b holds node t (local index).  For every layer l, tree b, kv head g
+ * and i = 0 .. accept_len[b]:
+ *   cache'[l][b][g][kv_len[b] + i][:] = cache[l][b][g][kv_len[b] + path[b][i]][:]
+ * computed from the cache as it was before the call (a destination row may
+ * be the source of another path entry; the kernel reads every moved row
+ * before it writes any).  kv_len_out[b] = kv_len[b] + accept_len[b] + 1.
+ * Rows of the tree past the new length are left as they were.
+ *
+ * Arguments as for adt_kv_compact, without the tree buffers;
+ * node_offsets[b+1] - node_offsets[b] is tree b's size n_b, and
+ * kv_len[b] + n_b <= max_kv.  1 <= max_path <= 256 (ADT_ERR_UNSUPPORTED
+ * above).  A path entry outside the tree, or a tree that does not fit,
+ * sets a device error bit and skips tree b.
+ * ------------------------------------------------------------------------ */
+adt_status adt_kv_compact_inplace(adt_bf16* k_cache, adt_bf16* v_cache, const int32_t* kv_len,
+                                  int32_t* kv_len_out, const int32_t* node_offsets,
+                                  const int32_t* path, int32_t max_path, const int32_t* accept_len,
+                                  int32_t B, int32_t Hkv, int32_t D, int32_t num_layers,
+                                  int32_t max_kv, int64_t cache_layer_stride,
+                                  int64_t cache_stride_b, int64_t cache_stride_h, void* stream);
+
+/* ------------------------------------------------------------------------
  * Depth / width controller (host only, no GPU).  Sec. 4.1 adjacent
  * initialisation, Eq. 2 bisectional adaptation, bounds at the end of
  * Sec. 4.2, hyper-parameters Sec. 5.1.  For the tree that emits grid

@@ -392,3 +392,21 @@ def kv_compact(k_cache, v_cache, kv_len, k_tree, v_tree, node_offsets, paths):
             vc[:, b, :, base + i, :] = v_tree[:, src, :, :]
         new_len[b] = base + len(path)
     return kc, vc, new_len
+
+
+def kv_compact_inplace(k_cache, v_cache, kv_len, paths):
+    """The cache holds tree b's K/V in its tail: row kv_len[b] + t is node t.
+    For every layer l, tree b and i in 0..a_b, computed from the cache as it
+    was before (Sec. 3.1: the accepted tokens extend the prefix):
+        cache'[l, b, :, kv_len[b] + i, :] = cache[l, b, :, kv_len[b] + path_b[i], :]
+    Returns (k_cache', v_cache', kv_len') as new arrays."""
+    kc = np.array(k_cache, copy=True)
+    vc = np.array(v_cache, copy=True)
+    new_len = np.array(kv_len, dtype=np.int64, copy=True)
+    for b, path in enumerate(paths):
+        base = int(kv_len[b])
+        for i, node in enumerate(path):
+            kc[:, b, :, base + i, :] = k_cache[:, b, :, base + int(node), :]
+            vc[:, b, :, base + i, :] = v_cache[:, b, :, base + int(node), :]
+        new_len[b] = base + len(path)
+    return kc, vc, new_len

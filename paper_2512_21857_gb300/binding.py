@@ -29,7 +29,7 @@ EXPORTED = [
     "adt_tree_expand_workspace_size", "adt_tree_expand", "adt_tree_expand_cfg",
     "adt_tree_rerank_workspace_size", "adt_tree_rerank",
     "adt_tree_accept_workspace_size", "adt_tree_accept", "adt_tree_accept_cfg",
-    "adt_kv_compact",
+    "adt_kv_compact", "adt_kv_compact_inplace",
     "adt_ctrl_create", "adt_ctrl_destroy", "adt_ctrl_next", "adt_ctrl_update", "adt_ctrl_get",
 ]
 
@@ -72,6 +72,8 @@ _SIGS = {
                              _F32, _P, _I32, _P, _P, _P, _SZ, _P], _I32),
     "adt_kv_compact": ([_P, _P, _P, _P, _P, _P, _P, _P, _I32, _P, _I32, _I32, _I32, _I32, _I32, _I64, _I64,
                         _I64, _I64, _P], _I32),
+    "adt_kv_compact_inplace": ([_P, _P, _P, _P, _P, _P, _I32, _P, _I32, _I32, _I32, _I32, _I32, _I64, _I64, _I64,
+                                _P], _I32),
     "adt_ctrl_create": ([ctypes.POINTER(CtrlParams), _I32, _I32, ctypes.POINTER(_P)], _I32),
     "adt_ctrl_destroy": ([_P], None),
     "adt_ctrl_next": ([_P, _I32, ctypes.POINTER(_I32), ctypes.POINTER(_I32)], _I32),
@@ -264,6 +266,16 @@ def adt_kv_compact(k_cache, v_cache, kv_len, kv_len_out, k_tree, v_tree, node_of
                               B, Hkv, D, num_layers, max_kv, cache_layer_stride, cache_stride_b, cache_stride_h,
                               tree_layer_stride, _stream(stream))
     _check(st, "adt_kv_compact")
+
+
+def adt_kv_compact_inplace(k_cache, v_cache, kv_len, kv_len_out, node_offsets, path, max_path, accept_len, *, B,
+                           Hkv, D, num_layers, max_kv, cache_layer_stride, cache_stride_b, cache_stride_h,
+                           stream=None) -> None:
+    st = lib().adt_kv_compact_inplace(_ptr(k_cache), _ptr(v_cache), _ptr(kv_len), _ptr(kv_len_out),
+                                      _ptr(node_offsets), _ptr(path), int(max_path), _ptr(accept_len), B, Hkv, D,
+                                      num_layers, max_kv, cache_layer_stride, cache_stride_b, cache_stride_h,
+                                      _stream(stream))
+    _check(st, "adt_kv_compact_inplace")
 
 
 # ----------------------------------------------------------------------------- controller

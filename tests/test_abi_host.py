@@ -68,6 +68,9 @@ def test_invalid_arguments_rejected_before_launch(lib):
     # compact: kv_len_out aliasing kv_len, unaligned stride
     assert lib.adt_kv_compact(f, f, f, f, f, f, f, f, 8, f, 1, 2, 64, 2, 100, 64, 64, 64, 64, None) == 1
     assert lib.adt_kv_compact(f, f, f, None, f, f, f, f, 8, f, 1, 2, 64, 2, 100, 65, 64, 64, 64, None) == 1
+    # in-place compact: more than 256 staged path rows -> unsupported; kv_len_out aliasing kv_len
+    assert lib.adt_kv_compact_inplace(f, f, f, None, f, f, 257, f, 1, 2, 64, 2, 300, 64, 64, 64, None) == 2
+    assert lib.adt_kv_compact_inplace(f, f, f, f, f, f, 8, f, 1, 2, 64, 2, 300, 64, 64, 64, None) == 1
 
 
 def _run_both(params, grid, accepts):

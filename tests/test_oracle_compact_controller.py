@@ -40,6 +40,47 @@ def test_compact_overflow_rejected():
         oracle.kv_compact(z, z, [2], zt, zt, [0, 3], [[0, 1]])
 
 
+def test_compact_inplace_hazard_path_brute_force():
+    """Tree in the cache tail, path [0, 2, 5]: row L + 2 is the destination
+    of entry 2 and the source of entry 1; every destination must get the
+    value its source had before the call."""
+    layers, B, Hkv, Lmax, D = 2, 1, 2, 16, 3
+    g = np.random.default_rng(1)
+    kc = g.standard_normal((layers, B, Hkv, Lmax, D))
+    vc = g.standard_normal((layers, B, Hkv, Lmax, D))
+    L = 4
+    k2, v2, nl = oracle.kv_compact_inplace(kc, vc, [L], [[0, 2, 5]])
+    assert nl.tolist() == [7]
+    assert (k2[:, 0, :, L] == kc[:, 0, :, L]).all()          # the root stays
+    assert (k2[:, 0, :, L + 1] == kc[:, 0, :, L + 2]).all()  # old row L + 2, before it is overwritten
+    assert (k2[:, 0, :, L + 2] == kc[:, 0, :, L + 5]).all()
+    assert (v2[:, 0, :, L + 2] == vc[:, 0, :, L + 5]).all()
+    rest = np.ones(Lmax, bool)
+    rest[L + 1:L + 3] = False
+    assert (k2[:, :, :, rest] == kc[:, :, :, rest]).all()
+
+
+def test_compact_inplace_equals_out_of_place_from_the_tail():
+    """The same commit through a separate tree buffer copied from the
+    cache tail gives the same cache."""
+    layers, B, Hkv, Lmax, D = 3, 2, 2, 20, 4
+    g = np.random.default_rng(2)
+    kc = g.standard_normal((layers, B, Hkv, Lmax, D))
+    vc = g.standard_normal((layers, B, Hkv, Lmax, D))
+    kv_len, sizes = [3, 9], [7, 6]
+    offs = np.concatenate([[0], np.cumsum(sizes)])
+    kt = np.concatenate([kc[:, b, :, kv_len[b]:kv_len[b] + sizes[b]].transpose(0, 2, 1, 3) for b in range(B)], 1)
+    vt = np.concatenate([vc[:, b, :, kv_len[b]:kv_len[b] + sizes[b]].transpose(0, 2, 1, 3) for b in range(B)], 1)
+    paths = [[0, 1, 3, 6], [0, 4, 5]]
+    a = oracle.kv_compact_inplace(kc, vc, kv_len, paths)
+    b = oracle.kv_compact(kc, vc, kv_len, kt, vt, offs, paths)
+    for x, y in zip(a, b):
+        assert np.array_equal(x, y)
+    # a = 0: nothing moves
+    same = oracle.kv_compact_inplace(kc, vc, kv_len, [[0], [0]])
+    assert np.array_equal(same[0], kc) and np.array_equal(same[1], vc) and same[2].tolist() == [4, 10]
+
+
 def test_splitmix64_published_vectors(golden_dir):
     g = json.load(open(os.path.join(golden_dir, "splitmix64.json")))
     for c in g["cases"]:

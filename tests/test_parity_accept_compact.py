@@ -175,3 +175,47 @@ def test_compact_overflow_skips_tree_and_flags():
     got = gkc.cpu()
     assert torch.equal(got[:, 0], kc[:, 0])  # tree 0 (8 + 3 > 10) untouched
     assert torch.equal(got[:, 1, :, 3], kt[:, 4])
+
+
+def _run_inplace(kc, vc, kv, sizes, paths, max_path=16, max_kv=None):
+    offs = np.concatenate([[0], np.cumsum(sizes)]).astype(np.int32)
+    parr = np.full((len(sizes), max_path), -1, np.int32)
+    for b, p in enumerate(paths):
+        parr[b, :len(p)] = p
+    alen = np.array([len(p) - 1 for p in paths], np.int32)
+    dev = "cuda"
+    gkc, gvc = kc.to(dev), vc.to(dev)
+    kv_out = torch.empty(len(sizes), dtype=torch.int32, device=dev)
+    layers, Bn, Hkv, Lmax, D = kc.shape
+    B.adt_kv_compact_inplace(gkc, gvc, i32(kv), kv_out, i32(offs), i32(parr), max_path, i32(alen), B=Bn, Hkv=Hkv,
+                             D=D, num_layers=layers, max_kv=Lmax if max_kv is None else max_kv,
+                             cache_layer_stride=kc.stride(0), cache_stride_b=kc.stride(1),
+                             cache_stride_h=kc.stride(2))
+    torch.cuda.synchronize()
+    return gkc.cpu(), gvc.cpu(), kv_out.cpu().numpy()
+
+
+@pytest.mark.parametrize("layers,sizes,Hkv,D,Lmax,kv,paths", [
+    (32, [64], 32, 128, 2470, [2400], [[0, 5, 17, 40, 41, 63]]),
+    (3, [26, 1, 9], 8, 64, 600, [512, 0, 590], [[0, 2, 11], [0], [0, 1, 2, 3, 4, 5, 6, 7, 8]]),
+    (2, [8], 4, 128, 32, [10], [[0, 2, 5]]),               # row L + 2 is written and also read
+    (2, [256], 2, 64, 300, [40], [list(range(0, 256, 17))]),  # 256-node tree, 16-entry path
+])
+def test_compact_inplace_matches_oracle(layers, sizes, Hkv, D, Lmax, kv, paths):
+    kc, vc, _, _ = _compact_inputs(layers, sizes, Hkv, D, Lmax, kv, seed=layers + D + 1)
+    gk, gv, gl = _run_inplace(kc, vc, kv, sizes, paths)
+    rk, rv, rl = oracle.kv_compact_inplace(kc.view(torch.int16).numpy(), vc.view(torch.int16).numpy(), kv, paths)
+    assert np.array_equal(gk.view(torch.int16).numpy(), rk)
+    assert np.array_equal(gv.view(torch.int16).numpy(), rv)
+    assert gl.tolist() == rl.tolist()
+
+
+def test_compact_inplace_rejects_bad_trees():
+    kc, vc, _, _ = _compact_inputs(2, [4, 4], 2, 64, 12, None, seed=2)
+    B.adt_get_device_error()
+    # tree 0: rows 9 .. 12 do not fit in 12; tree 1: path entry 4 is outside its 4 nodes
+    gk, gv, gl = _run_inplace(kc, vc, [9, 2], [4, 4], [[0, 1], [0, 4]])
+    bits = B.adt_get_device_error()
+    assert bits & B.DEVERR_KV_RANGE and bits & B.DEVERR_BAD_PATH
+    assert gl.tolist() == [9, 2]
+    assert torch.equal(gk, kc) and torch.equal(gv, vc)
