@@ -374,6 +374,11 @@ adt_status adt_kv_compact_inplace(adt_bf16* k_cache, adt_bf16* v_cache, const in
  *         vertical: of the tree that emitted pos-W, horizontal if i = 0 or
  *         not generated; random: d ~ U{d_lo..d_hi}, k ~ U{k_lo..k_hi} from
  *         SplitMix64(seed + c*0x9E3779B97F4A7C15), c = 2*pos (d), 2*pos+1 (k);
+ *         tokenflock (the Table 3 alternative): the weighted mean over the
+ *         generated positions q < pos within distance delta = flock_delta,
+ *         (x_q - x)^2 + (y_q - y)^2 <= delta^2 (x column, y row), with
+ *         weights delta + 1 - (y - y_q) (the paper's (delta - dy + 1)/delta,
+ *         normalised), rounded half up;
  *         (d0, k0) when nothing precedes; fix_d / fix_k > 0 override.
  *   adapt alpha = a / d of the previous tree: alpha >= beta -> (d+l_d, k-l_k),
  *         else (d-l_d, k+l_k); no adaptation for an image's first tree.
@@ -381,7 +386,7 @@ adt_status adt_kv_compact_inplace(adt_bf16* k_cache, adt_bf16* v_cache, const in
  *         adapted depth exceeds 1, else to [1, k_cap].
  * The paper's open bounds (0,10) / (3,14) are the closed [1,9] / [4,13].
  * ------------------------------------------------------------------------ */
-enum { ADT_INIT_HORIZONTAL = 0, ADT_INIT_VERTICAL = 1, ADT_INIT_RANDOM = 2 };
+enum { ADT_INIT_HORIZONTAL = 0, ADT_INIT_VERTICAL = 1, ADT_INIT_RANDOM = 2, ADT_INIT_TOKENFLOCK = 3 };
 
 typedef struct adt_ctrl_params {
   double beta;
@@ -393,13 +398,14 @@ typedef struct adt_ctrl_params {
   int32_t k_cap;
   int32_t fix_d, fix_k;
   uint64_t seed;
+  int32_t flock_delta; /* tokenflock neighbourhood radius, >= 1 */
 } adt_ctrl_params;
 
 typedef struct adt_ctrl adt_ctrl; /* opaque; one per image */
 
 /* Creates a controller for a grid_h x grid_w token grid.  Checks
  * 1 <= d_lo <= d_hi, 1 <= k_lo <= k_hi <= k_cap, l_d, l_k >= 0, d0, k0 >= 1,
- * grid sizes >= 1.  *out receives a heap object freed by adt_ctrl_destroy. */
+ * 1 <= flock_delta <= 64 for tokenflock, grid sizes >= 1.  *out receives a heap object freed by adt_ctrl_destroy. */
 adt_status adt_ctrl_create(const adt_ctrl_params* params, int32_t grid_h, int32_t grid_w,
                            adt_ctrl** out);
 void adt_ctrl_destroy(adt_ctrl* ctrl);

@@ -9,6 +9,13 @@ Per image, for the draft tree that will emit grid position pos = (i, j):
        vertical repeat   - the tree that emitted (i-1, j); horizontal when
                            i = 0 or that position is not generated yet;
        random            - d~ ~ U{d_lo..d_hi}, k~ ~ U{k_lo..k_hi};
+       TokenFlock        - (the alternative of Table 3) the set Omega of
+                           generated positions t_j before pos within
+                           Euclidean distance delta, x the column and y the
+                           row; d~ = sum d_j w_j / sum w_j with
+                           w_j = (delta - (y_i - y_j) + 1) / delta (norm()
+                           read as dividing by the sum of the weights), k~
+                           likewise, each rounded half up;
      the first tree of an image uses (d0, k0); fix_d / fix_k pin d~ / k~
      (the fixed-value ablations of Table 3).
   2. bisect with the acceptance rate alpha = a / d of the previous tree
@@ -26,10 +33,12 @@ Random initialisation draws from SplitMix64 (Steele, Lea and Flood, OOPSLA
 from __future__ import annotations
 
 from dataclasses import dataclass, field
+from fractions import Fraction
 
 INIT_HORIZONTAL = 0
 INIT_VERTICAL = 1
 INIT_RANDOM = 2
+INIT_TOKENFLOCK = 3
 
 _MASK = (1 << 64) - 1
 _GAMMA = 0x9E3779B97F4A7C15
@@ -64,6 +73,7 @@ class CtrlParams:
     fix_d: int = 0
     fix_k: int = 0
     seed: int = 0
+    flock_delta: int = 2
 
 
 def anole_params(**kw) -> CtrlParams:
@@ -101,7 +111,10 @@ class Controller:
         if not (0 <= pos < n):
             raise ValueError("pos outside the grid")
         i = pos // self.grid_w
-        if P.init_mode == INIT_RANDOM:
+        flock = self._flock(pos) if P.init_mode == INIT_TOKENFLOCK else None
+        if P.init_mode == INIT_TOKENFLOCK:
+            d_t, k_t = flock if flock is not None else (P.d0, P.k0)
+        elif P.init_mode == INIT_RANDOM:
             d_t = P.d_lo + counter_draw(P.seed, 2 * pos) % (P.d_hi - P.d_lo + 1)
             k_t = P.k_lo + counter_draw(P.seed, 2 * pos + 1) % (P.k_hi - P.k_lo + 1)
         elif P.init_mode == INIT_VERTICAL and i >= 1 and self.d_grid[pos - self.grid_w] > 0:
@@ -125,6 +138,25 @@ class Controller:
         k = _clamp(k, P.k_lo, P.k_hi) if restrict_k else _clamp(k, 1, P.k_cap)
         self.cur = (d, k)
         return d, k
+
+    def _flock(self, pos: int):
+        """TokenFlock's weighted mean over Omega (exact fractions, rounded
+        half up), or None when Omega is empty."""
+        delta = self.params.flock_delta
+        y_i, x_i = divmod(pos, self.grid_w)
+        num_d, num_k, den = Fraction(0), Fraction(0), Fraction(0)
+        for q in range(pos):  # j < i: the positions generated before
+            y_j, x_j = divmod(q, self.grid_w)
+            if (x_i - x_j) ** 2 + (y_i - y_j) ** 2 > delta ** 2 or self.d_grid[q] == 0:
+                continue
+            w = Fraction(delta - (y_i - y_j) + 1, delta)
+            num_d += self.d_grid[q] * w
+            num_k += self.k_grid[q] * w
+            den += w
+        if den == 0:
+            return None
+        half_up = lambda f: (f + Fraction(1, 2)).__floor__()
+        return half_up(num_d / den), half_up(num_k / den)
 
     def update(self, pos: int, accept_len: int) -> int:
         """Record the tree that just verified: alpha = a / d (Sec. 3.2), and

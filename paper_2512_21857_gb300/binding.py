@@ -20,7 +20,7 @@ ADT_OK = 0
 STATUS_NAMES = {0: "ADT_OK", 1: "ADT_ERR_INVALID_ARG", 2: "ADT_ERR_UNSUPPORTED", 3: "ADT_ERR_CUDA",
                 4: "ADT_ERR_TIMEOUT", 5: "ADT_ERR_WORKSPACE", 6: "ADT_ERR_DEVICE"}
 ACCEPT_GREEDY, ACCEPT_SPEC, ACCEPT_SPEC_DET = 0, 1, 2
-INIT_HORIZONTAL, INIT_VERTICAL, INIT_RANDOM = 0, 1, 2
+INIT_HORIZONTAL, INIT_VERTICAL, INIT_RANDOM, INIT_TOKENFLOCK = 0, 1, 2, 3
 DEVERR_BAD_TREE, DEVERR_KV_RANGE, DEVERR_BAD_PATH, DEVERR_TIMEOUT, DEVERR_BAD_INDEX = 1, 2, 4, 8, 16
 
 EXPORTED = [
@@ -45,7 +45,8 @@ class CtrlParams(ctypes.Structure):
                 ("d_lo", ctypes.c_int32), ("d_hi", ctypes.c_int32), ("k_lo", ctypes.c_int32),
                 ("k_hi", ctypes.c_int32), ("init_mode", ctypes.c_int32), ("d0", ctypes.c_int32),
                 ("k0", ctypes.c_int32), ("clamp_k_always", ctypes.c_int32), ("k_cap", ctypes.c_int32),
-                ("fix_d", ctypes.c_int32), ("fix_k", ctypes.c_int32), ("seed", ctypes.c_uint64)]
+                ("fix_d", ctypes.c_int32), ("fix_k", ctypes.c_int32), ("seed", ctypes.c_uint64),
+                ("flock_delta", ctypes.c_int32)]
 
 
 _P, _I32, _I64, _F32, _SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
@@ -285,9 +286,9 @@ class Controller:
 
     def __init__(self, grid_h, grid_w, *, beta=1.0, l_d=1, l_k=3, d_lo=1, d_hi=9, k_lo=4, k_hi=13,
                  init_mode=INIT_HORIZONTAL, d0=5, k0=10, clamp_k_always=True, k_cap=64, fix_d=0, fix_k=0,
-                 seed=0):
+                 seed=0, flock_delta=2):
         self._p = CtrlParams(beta, l_d, l_k, d_lo, d_hi, k_lo, k_hi, init_mode, d0, k0, int(bool(clamp_k_always)),
-                             k_cap, fix_d, fix_k, seed)
+                             k_cap, fix_d, fix_k, seed, flock_delta)
         h = ctypes.c_void_p()
         _check(lib().adt_ctrl_create(ctypes.byref(self._p), grid_h, grid_w, ctypes.byref(h)), "adt_ctrl_create")
         self._h = h

@@ -33,6 +33,36 @@ uint64_t counter_draw(uint64_t seed, uint64_t counter) { return splitmix64(seed 
 
 int32_t clamp(int32_t x, int32_t lo, int32_t hi) { return x < lo ? lo : (x > hi ? hi : x); }
 
+// TokenFlock initialisation (the alternative of Table 3): the generated
+// positions within Euclidean distance delta of (row i, column j) that come
+// before it, each weighted by delta + 1 - (rows above); returns false when
+// there are none.  Integer weights make the mean an exact fraction, rounded
+// half up.
+bool flock_init(const adt_ctrl* c, int32_t i, int32_t j, int32_t* d, int32_t* k) {
+  const int32_t delta = c->p.flock_delta;
+  int64_t wsum = 0, dsum = 0, ksum = 0;
+  for (int32_t dy = delta; dy >= 0; --dy) {
+    const int32_t r = i - dy;
+    if (r < 0) continue;
+    for (int32_t dx = -delta; dx <= delta; ++dx) {
+      const int32_t col = j + dx;
+      if (col < 0 || col >= c->w) continue;
+      if (dy == 0 && dx >= 0) break;  // only positions before (i, j)
+      if (dx * dx + dy * dy > delta * delta) continue;
+      const int32_t q = r * c->w + col;
+      if (c->d_grid[q] <= 0) continue;
+      const int64_t wgt = delta + 1 - dy;
+      wsum += wgt;
+      dsum += wgt * c->d_grid[q];
+      ksum += wgt * c->k_grid[q];
+    }
+  }
+  if (wsum == 0) return false;
+  *d = static_cast<int32_t>((2 * dsum + wsum) / (2 * wsum));
+  *k = static_cast<int32_t>((2 * ksum + wsum) / (2 * wsum));
+  return true;
+}
+
 }  // namespace
 
 extern "C" {
@@ -43,8 +73,10 @@ adt_status adt_ctrl_create(const adt_ctrl_params* params, int32_t grid_h, int32_
   const adt_ctrl_params& p = *params;
   if (p.d_lo < 1 || p.d_hi < p.d_lo || p.k_lo < 1 || p.k_hi < p.k_lo || p.k_cap < p.k_hi) return ADT_ERR_INVALID_ARG;
   if (p.l_d < 0 || p.l_k < 0 || p.d0 < 1 || p.k0 < 1 || p.fix_d < 0 || p.fix_k < 0) return ADT_ERR_INVALID_ARG;
-  if (p.init_mode != ADT_INIT_HORIZONTAL && p.init_mode != ADT_INIT_VERTICAL && p.init_mode != ADT_INIT_RANDOM)
+  if (p.init_mode != ADT_INIT_HORIZONTAL && p.init_mode != ADT_INIT_VERTICAL && p.init_mode != ADT_INIT_RANDOM &&
+      p.init_mode != ADT_INIT_TOKENFLOCK)
     return ADT_ERR_INVALID_ARG;
+  if (p.init_mode == ADT_INIT_TOKENFLOCK && (p.flock_delta < 1 || p.flock_delta > 64)) return ADT_ERR_INVALID_ARG;
   if (static_cast<int64_t>(grid_h) * grid_w > (int64_t{1} << 28)) return ADT_ERR_INVALID_ARG;
   adt_ctrl* c = new (std::nothrow) adt_ctrl;
   if (!c) return ADT_ERR_INVALID_ARG;
@@ -72,7 +104,12 @@ adt_status adt_ctrl_next(adt_ctrl* c, int32_t pos, int32_t* depth, int32_t* widt
   const int32_t i = pos / c->w;
   int32_t d, k;
   // Adjacent initialisation (Sec. 4.1).
-  if (P.init_mode == ADT_INIT_RANDOM) {
+  if (P.init_mode == ADT_INIT_TOKENFLOCK) {
+    if (!flock_init(c, i, pos % c->w, &d, &k)) {
+      d = P.d0;
+      k = P.k0;
+    }
+  } else if (P.init_mode == ADT_INIT_RANDOM) {
     d = P.d_lo + static_cast<int32_t>(counter_draw(P.seed, 2ull * static_cast<uint64_t>(pos)) %
                                       static_cast<uint64_t>(P.d_hi - P.d_lo + 1));
     k = P.k_lo + static_cast<int32_t>(counter_draw(P.seed, 2ull * static_cast<uint64_t>(pos) + 1) %

@@ -92,7 +92,7 @@ def _run_both(params, grid, accepts):
         assert ctl_c.get(p) == (ctl_o.d_grid[p], ctl_o.k_grid[p])
 
 
-@pytest.mark.parametrize("init_mode", [0, 1, 2])
+@pytest.mark.parametrize("init_mode", [0, 1, 2, 3])
 @pytest.mark.parametrize("preset", ["anole", "llamagen", "c4"])
 def test_controller_matches_oracle_bit_exactly(lib, init_mode, preset):
     params = {
@@ -107,6 +107,9 @@ def test_controller_matches_oracle_bit_exactly(lib, init_mode, preset):
     _run_both(dict(params, clamp_k_always=False, k_cap=64), (24, 24), accepts)
     _run_both(dict(params, fix_d=1, fix_k=25 if preset == "llamagen" else 0), (8, 8), accepts)
     _run_both(dict(params, beta=0.5), (8, 8), accepts)
+    if init_mode == 3:
+        for delta in (1, 3, 5):
+            _run_both(dict(params, flock_delta=delta), (24, 24), accepts)
 
 
 def test_controller_hand_traces_through_abi(lib, golden_dir):
@@ -124,6 +127,8 @@ def test_controller_hand_traces_through_abi(lib, golden_dir):
 def test_controller_rejects_bad_input(lib):
     with pytest.raises(B.AdtError):
         B.Controller(4, 4, d_lo=3, d_hi=2)
+    with pytest.raises(B.AdtError):
+        B.Controller(4, 4, init_mode=B.INIT_TOKENFLOCK, flock_delta=0)
     c = B.Controller(4, 4)
     with pytest.raises(B.AdtError):
         c.update(0, 1)  # update before next

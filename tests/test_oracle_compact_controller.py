@@ -139,3 +139,43 @@ def test_controller_rejects_bad_accept_len():
     c.next(0)
     with pytest.raises(ValueError):
         c.update(0, 6)
+
+
+def test_tokenflock_hand_examples():
+    """TokenFlock (Table 3's alternative initialisation): Omega = generated
+    positions before (i, j) within distance delta; weights delta + 1 - dy,
+    normalised; the means rounded half up."""
+    P = oracle.CtrlParams(init_mode=oracle.INIT_TOKENFLOCK, flock_delta=1)
+    c = oracle.Controller(P, 3, 4)
+    # (1, 1) with delta 1: left neighbour (1, 0) weight 2, (0, 1) above weight 1
+    c.d_grid[:5] = [9, 3, 9, 9, 6]
+    c.k_grid[:5] = [13, 10, 13, 13, 4]
+    assert c._flock(5) == (5, 6)          # (2*6 + 3) / 3, (2*4 + 10) / 3
+    # delta 2 at (0, 2): (0, 0) and (0, 1), both weight 3: means 4.5 and 11.5 round up
+    c2 = oracle.Controller(oracle.CtrlParams(init_mode=oracle.INIT_TOKENFLOCK, flock_delta=2), 2, 8)
+    c2.d_grid[:2] = [4, 5]
+    c2.k_grid[:2] = [10, 13]
+    assert c2._flock(2) == (5, 12)
+    # delta 2 at (2, 2) of a 4 x 5 grid: same row (2,0),(2,1) weight 3; row 1
+    # columns 1..3 weight 2; (0, 2) weight 1 -> sum of weights 13
+    c3 = oracle.Controller(oracle.CtrlParams(init_mode=oracle.INIT_TOKENFLOCK, flock_delta=2), 4, 5)
+    d = [1, 2, 3, 4, 5, 6, 7, 8, 9, 1, 2, 3]
+    c3.d_grid[:12] = d
+    c3.k_grid[:12] = [4] * 12
+    num = 3 * d[10] + 3 * d[11] + 2 * (d[6] + d[7] + d[8]) + 1 * d[2]   # = 6 + 9 + 48 + 3 = 66
+    assert num == 66 and c3._flock(12) == (5, 4)                        # 66 / 13 = 5.08 -> 5
+    # nothing generated before: (d0, k0)
+    assert oracle.Controller(P, 3, 4)._flock(0) is None
+
+
+def test_tokenflock_trace():
+    P = oracle.anole_params(init_mode=oracle.INIT_TOKENFLOCK, flock_delta=2)
+    c = oracle.Controller(P, 4, 8)
+    assert c.next(0) == (5, 10)           # first tree: (d0, k0), no adaptation
+    assert c.update(0, 2) == 3            # alpha = 2/5 < beta
+    # Omega of (0, 3): (0, 1) and (0, 2), both (5, 10) -> (5, 10); alpha < 1 -> (4, 13)
+    assert c.next(3) == (4, 13)
+    assert c.update(3, 4) == 8            # alpha = 1 >= beta; positions 3..7 hold (4, 13)
+    # Omega of (1, 0): (0, 0) .. (0, 2)? distance <= 2 -> (0, 0) w 2, (0, 1) w 2, and
+    # (0, 2) is at distance sqrt(5) > 2: mean of (5, 10) twice = (5, 10); alpha >= 1 -> (6, 7)
+    assert c.next(8) == (6, 7)

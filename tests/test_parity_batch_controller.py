@@ -29,7 +29,8 @@ def _bits(t):
     return t.contiguous().view(torch.int16).cpu().numpy()
 
 
-def test_ragged_batch_three_controller_steps():
+@pytest.mark.parametrize("init_mode", [B.INIT_HORIZONTAL, B.INIT_TOKENFLOCK])
+def test_ragged_batch_three_controller_steps(init_mode):
     ensure_built()
     nb, layers, H, D, V, steps, seed = 8, 2, 8, 128, 16384, 3, 404
     g = synth.rng(seed, "batch_controller")
@@ -37,8 +38,9 @@ def test_ragged_batch_three_controller_steps():
     pos = [int(x) for x in g.integers(0, GRID[0] * GRID[1] - 100, size=nb)]
     amap = synth.acceptance_map(*GRID, seed).ravel()
     lmax = 2400 + steps * 11 + 64
-    ctl_c = [B.Controller(*GRID, **PARAMS, seed=seed + b) for b in range(nb)]
-    ctl_o = [oracle.Controller(oracle.CtrlParams(**PARAMS, seed=seed + b), *GRID) for b in range(nb)]
+    ctl_c = [B.Controller(*GRID, **PARAMS, init_mode=init_mode, seed=seed + b) for b in range(nb)]
+    ctl_o = [oracle.Controller(oracle.CtrlParams(**PARAMS, init_mode=init_mode, seed=seed + b), *GRID)
+             for b in range(nb)]
     kc = vc = None  # the committed caches (bf16 bits), carried to the next step
     seen_dk, seen_a = set(), []
     B.adt_get_device_error()
