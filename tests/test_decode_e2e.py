@@ -1,0 +1,71 @@
+"""The end-to-end decode loop (random-init target, EAGLE-style draft head,
+ADT-Tree trees every step) against vanilla greedy decoding with the same
+target: greedy verification is lossless, so both must emit the same tokens.
+The two run different launch shapes (a tree of up to 64 nodes vs one node,
+batched GEMMs of different sizes), so their logits agree only to rounding;
+a difference is allowed only where vanilla decoding itself faced a near tie
+(top-2 logit gap below 0.05), and the comparison stops there."""
+import pytest
+import torch
+
+from gpu_cases import ensure_built
+from paper_2512_21857_gb300 import binding as B
+from paper_2512_21857_gb300.decode import Decoder, DecoderWeights, ModelShape, greedy_decode
+
+pytestmark = pytest.mark.gpu
+NEAR_TIE = 0.05
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    ensure_built()
+
+
+def _compare(adt, ref, margins):
+    """Tokens equal up to the end, or up to a near tie of the reference."""
+    for i, (a, r) in enumerate(zip(adt, ref)):
+        if a != r:
+            assert margins[i] < NEAR_TIE, f"token {i}: {a} != {r} with a top-2 gap of {margins[i]:.3f}"
+            return i
+    assert len(adt) == len(ref)
+    return len(adt)
+
+
+def _prompt(vocab, n, seed):
+    g = torch.Generator().manual_seed(seed)
+    return torch.randint(0, vocab, (n,), generator=g).tolist()
+
+
+SMALL = ModelShape(layers=2, hidden=256, heads=2, kv_heads=2, head_dim=128, ffn=512, vocab=4096, init_std=0.1,
+                  lm_std=1.0)
+
+
+@pytest.mark.parametrize("batch", [1, 2])
+def test_adt_decode_equals_greedy(batch):
+    dec = Decoder(SMALL, batch=batch, grid=(8, 8), prompt_len=8, seed=7, max_nodes=64)
+    prompt = _prompt(SMALL.vocab, 8, 1)
+    out, stats = dec.generate(prompt)
+    ref, margins = greedy_decode(SMALL, dec.target_w, prompt, 64, batch=batch, return_margins=True)
+    for b in range(batch):
+        assert len(out[b]) == 64
+        n = _compare(out[b], ref[b], margins[b])
+        assert n >= 16, f"image {b}: only {n} tokens before a near tie"
+    assert B.adt_get_device_error() == 0
+    assert stats.steps >= 1 and stats.tau >= 1.0
+
+
+def test_adt_decode_with_a_draft_that_matches_the_target():
+    """A one-layer target whose draft head reproduces it: trees are accepted
+    deep (long paths through accept and both K/V commits), and the output
+    is still vanilla greedy's."""
+    shape = ModelShape(layers=1, hidden=256, heads=2, kv_heads=2, head_dim=128, ffn=512, vocab=4096, init_std=0.1,
+                       lm_std=1.0)
+    dec = Decoder(shape, batch=1, grid=(8, 12), prompt_len=8, seed=11, max_nodes=64, draft_equals_target=True,
+                  ctrl_params=dict(d_lo=1, d_hi=6, k_lo=2, k_hi=4))
+    prompt = _prompt(shape.vocab, 8, 2)
+    out, stats = dec.generate(prompt)
+    ref, margins = greedy_decode(shape, dec.target_w, prompt, 96, return_margins=True)
+    n = _compare(out[0], ref[0], margins[0])
+    assert n >= 24
+    assert stats.accepted >= stats.steps, "a matching draft should average at least one accepted token per step"
+    assert B.adt_get_device_error() == 0
