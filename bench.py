@@ -393,6 +393,51 @@ def cpu_sample_main(args):
 
 # ------------------------------------------------------------------ main
 
+def run_decode(args):
+    """The end-to-end synthetic decode loop (random-init 7B-shape target and
+    a one-layer EAGLE-style draft head, ADT-Tree trees every step) over a
+    square image-token grid, timed as a whole, next to vanilla greedy
+    decoding of the same tokens with the same target.  One JSON line."""
+    import torch
+    from paper_2512_21857_gb300 import binding as B
+    from paper_2512_21857_gb300 import build
+    from paper_2512_21857_gb300.decode import Decoder, ModelShape, greedy_decode
+    build.build()
+    B.lib()
+    shape = ModelShape(dtype=torch.float32) if args.decode_fp32 else ModelShape()
+    g = args.decode_grid
+    prompt = [int(x) for x in torch.randint(0, shape.vocab, (16,), generator=torch.Generator().manual_seed(7))]
+    dec = Decoder(shape, batch=args.decode_batch, grid=(g, g), prompt_len=16, seed=2025)
+    # warm-up: a small grid with the same weights (cuBLAS plans, library set-up)
+    Decoder(shape, batch=args.decode_batch, grid=(4, 4), prompt_len=16, seed=2025,
+            target=dec.target_w).generate(prompt)
+    out, st = dec.generate(prompt)
+    n = g * g
+    t0 = time.perf_counter()
+    ref, margins = greedy_decode(shape, dec.target_w, prompt, n, batch=args.decode_batch, return_margins=True)
+    torch.cuda.synchronize()
+    t_van = time.perf_counter() - t0
+    same = sum(1 for b in range(args.decode_batch) for x, y in zip(out[b], ref[b]) if x == y)
+    diffs = [next((i for i, (x, y) in enumerate(zip(out[b], ref[b])) if x != y), n) for b in range(args.decode_batch)]
+    first_diff = min(diffs)
+    # the greedy decision there, as a top-2 gap over the logit row's spread (a near tie when tiny)
+    gaps = [margins[b][diffs[b]] for b in range(args.decode_batch) if diffs[b] < n]
+    line = {"metric": "synthetic end-to-end decode tokens/s", "value": st.tokens / st.seconds, "unit": "tokens/s",
+            "n_gpus": 1, "higher_is_better": True, "dtype": "bf16", "data": "synthetic (random-init weights)",
+            "config": {"workload": f"random-init 7B-shape target (32 layers, hidden 4096, 32 heads x 128, SwiGLU "
+                                   f"11008, vocab 65536) + one-layer EAGLE-style draft head, {g}x{g} image tokens "
+                                   f"after a 16-token prompt, ADT-Tree controller (Anole bounds), greedy",
+                       "batch": args.decode_batch,
+                       "dense_dtype": "fp32" if args.decode_fp32 else "bf16"},
+            "tau": st.tau, "accepted_draft_tokens": st.accepted, "verify_steps": st.steps,
+            "mean_depth": st.mean_depth, "seconds": st.seconds,
+            "vanilla_greedy_tokens_per_s": args.decode_batch * n / t_van,
+            "speedup_vs_vanilla": (st.tokens / st.seconds) / (args.decode_batch * n / t_van),
+            "tokens_equal_to_vanilla_before_first_difference": first_diff, "tokens_equal_total": same,
+            "vanilla_relative_top2_gap_at_first_difference": max(gaps) if gaps else None}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -408,7 +453,14 @@ def main():
     ap.add_argument("--cpu-layers", type=int, default=1)
     ap.add_argument("--cpu-rows", type=int, default=1)
     ap.add_argument("--cpu-reps", type=int, default=1)
+    ap.add_argument("--decode", action="store_true", help="the end-to-end synthetic decode loop instead")
+    ap.add_argument("--decode-batch", type=int, default=1)
+    ap.add_argument("--decode-grid", type=int, default=48)
+    ap.add_argument("--decode-fp32", action="store_true", help="fp32 weights and residual stream in the harness")
     args = ap.parse_args()
+    if args.decode:
+        run_decode(args)
+        return
     if args.cpu_sample:
         cpu_sample_main(args)
         return

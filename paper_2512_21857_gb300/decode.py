@@ -48,6 +48,7 @@ class ModelShape:
     eps: float = 1e-5
     init_std: float = 0.02
     lm_std: float = 0.0        # LM head init std (0: init_std)
+    dtype: torch.dtype = torch.bfloat16  # weights and residual stream (the caches and attention stay bf16)
 
 
 def _rms_norm(x, w, eps):
@@ -74,7 +75,7 @@ class DecoderWeights:
         g = torch.Generator(device=device).manual_seed(seed)  # drawn on the device: 7B weights in seconds
         s = shape
         std = s.init_std
-        bf = dict(dtype=torch.bfloat16)
+        bf = dict(dtype=s.dtype)
 
         def rnd(*size, scale=std):
             return (torch.randn(*size, generator=g, device=device) * scale).to(**bf)
@@ -96,7 +97,7 @@ def lm_logits(weights: DecoderWeights, h, eps):
     """fp32 logits of hidden states h: final RMSNorm, then the LM head in
     fp32 (bf16 logits tie too often for a greedy argmax)."""
     if getattr(weights, "lm_head32", None) is None:
-        weights.lm_head32 = weights.lm_head.float()
+        weights.lm_head32 = weights.lm_head.float()  # the same tensor when the weights are fp32
     return _rms_norm(h, weights.norm, eps).float() @ weights.lm_head32
 
 
@@ -134,7 +135,7 @@ class TreeModel:
         for li, lw in enumerate(self.w.layers):
             h = _rms_norm(x, lw["ln1"], s.eps)
             qkv = h @ lw["wqkv"]
-            q = _rope(qkv[:, :hq].view(N, s.heads, s.head_dim), pos, s.rope_theta).contiguous()
+            q = _rope(qkv[:, :hq].view(N, s.heads, s.head_dim), pos, s.rope_theta).to(torch.bfloat16).contiguous()
             k_tree[li] = _rope(qkv[:, hq:hq + hk].view(N, s.kv_heads, s.head_dim), pos, s.rope_theta)
             v_tree[li] = qkv[:, hq + hk:].view(N, s.kv_heads, s.head_dim)
             B.adt_tree_attn(q, self.k_cache[li, sl], self.v_cache[li, sl], kv_len, k_tree[li], v_tree[li], parents,
@@ -142,7 +143,7 @@ class TreeModel:
                             max_nodes=self.max_nodes, max_kv=self.lmax, softmax_scale=s.head_dim ** -0.5, out=out,
                             workspace=self.ws, cache_stride_b=self.k_cache.stride(1),
                             cache_stride_h=self.k_cache.stride(2))
-            x = x + out.view(N, hq) @ lw["wo"]
+            x = x + out.view(N, hq).to(x.dtype) @ lw["wo"]
             h = _rms_norm(x, lw["ln2"], s.eps)
             gu = h @ lw["wgu"]
             x = x + (torch.nn.functional.silu(gu[:, : s.ffn].float()) * gu[:, s.ffn:].float()).to(x.dtype) @ lw["wd"]
@@ -208,7 +209,7 @@ class Decoder:
             # embedding through, and the layer is the target's
             dw = DecoderWeights(s, 0, seed + 1, device, lm=False, draft_fc=True)
             dw.layers = tw.layers[:1]
-            eye = torch.eye(s.hidden, dtype=torch.bfloat16, device=device)
+            eye = torch.eye(s.hidden, dtype=s.dtype, device=device)
             dw.fc = torch.cat([eye, torch.zeros_like(eye)], 0)
         else:
             dw = DecoderWeights(s, 1, seed + 1, device, lm=False, draft_fc=True)
@@ -255,7 +256,7 @@ class Decoder:
         kv_out = torch.empty(Bn, dtype=torch.int32, device=dev)
         self.target.commit(kt, vt, zero, kv_out, offs, path, n, alen, Bn)
         feats = h.view(Bn, n, s.hidden)
-        zf = torch.zeros(s.hidden, dtype=torch.bfloat16, device=dev)
+        zf = torch.zeros(s.hidden, dtype=s.dtype, device=dev)
         state = []
         for b in range(Bn):
             # the draft catches up on prompt[:-1]: parent features f_{t-1} (zeros for t = 0)
@@ -416,7 +417,8 @@ def greedy_decode(shape: ModelShape, weights: DecoderWeights, prompt, n_tokens, 
                   return_margins=False):
     """Vanilla greedy decoding with the same target: one node per step (a
     tree of its root alone).  Returns the tokens (and, with return_margins,
-    the top-1 minus top-2 logit gap of every decision)."""
+    the top-1 minus top-2 logit gap of every decision over the standard
+    deviation of that logit row)."""
     if not 2 <= len(prompt) <= 257:
         raise ValueError("prompt of 2 .. 257 tokens (the prefill is one tree)")
     model = TreeModel(shape, weights, batch, len(prompt) + n_tokens + 16, len(prompt) - 1, device)
@@ -449,7 +451,7 @@ def greedy_decode(shape: ModelShape, weights: DecoderWeights, prompt, n_tokens, 
         kv = kv_out.clone()
         out.append(nxt)
         if return_margins:
-            margins.append(top2.values[:, 0] - top2.values[:, 1])
+            margins.append((top2.values[:, 0] - top2.values[:, 1]) / logits.std(dim=-1))
         root = nxt
     toks = torch.stack(out, 1).cpu().tolist()
     if return_margins:

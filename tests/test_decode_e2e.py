@@ -4,7 +4,9 @@ target: greedy verification is lossless, so both must emit the same tokens.
 The two run different launch shapes (a tree of up to 64 nodes vs one node,
 batched GEMMs of different sizes), so their logits agree only to rounding;
 a difference is allowed only where vanilla decoding itself faced a near tie
-(top-2 logit gap below 0.05), and the comparison stops there."""
+(top-2 logit gap below 1 % of the logit row's standard deviation: a bf16
+residual stream moves logits of spread s by about s / 2^8 between the two
+shapes), and the comparison stops there."""
 import pytest
 import torch
 
@@ -13,7 +15,7 @@ from paper_2512_21857_gb300 import binding as B
 from paper_2512_21857_gb300.decode import Decoder, DecoderWeights, ModelShape, greedy_decode
 
 pytestmark = pytest.mark.gpu
-NEAR_TIE = 0.05
+NEAR_TIE = 0.01  # of the logit row's standard deviation
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -25,7 +27,7 @@ def _compare(adt, ref, margins):
     """Tokens equal up to the end, or up to a near tie of the reference."""
     for i, (a, r) in enumerate(zip(adt, ref)):
         if a != r:
-            assert margins[i] < NEAR_TIE, f"token {i}: {a} != {r} with a top-2 gap of {margins[i]:.3f}"
+            assert margins[i] < NEAR_TIE, f"token {i}: {a} != {r} with a relative top-2 gap of {margins[i]:.4f}"
             return i
     assert len(adt) == len(ref)
     return len(adt)
@@ -68,4 +70,19 @@ def test_adt_decode_with_a_draft_that_matches_the_target():
     n = _compare(out[0], ref[0], margins[0])
     assert n >= 24
     assert stats.accepted >= stats.steps, "a matching draft should average at least one accepted token per step"
+    assert B.adt_get_device_error() == 0
+
+
+def test_adt_decode_equals_greedy_fp32_stream():
+    """Eight layers with an fp32 residual stream and fp32 projections (the
+    caches and the library's attention stay bf16): the two launch shapes
+    then differ only by accumulation order, and the whole grid matches."""
+    shape = ModelShape(layers=8, hidden=512, heads=4, kv_heads=4, head_dim=128, ffn=1024, vocab=8192, init_std=0.05,
+                       lm_std=0.5, dtype=torch.float32)
+    dec = Decoder(shape, batch=2, grid=(8, 8), prompt_len=12, seed=5, max_nodes=64)
+    prompt = _prompt(shape.vocab, 12, 3)
+    out, stats = dec.generate(prompt)
+    ref, margins = greedy_decode(shape, dec.target_w, prompt, 64, batch=2, return_margins=True)
+    for b in range(2):
+        assert _compare(out[b], ref[b], margins[b]) >= 48
     assert B.adt_get_device_error() == 0
