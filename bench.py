@@ -407,14 +407,16 @@ def run_decode(args):
     shape = ModelShape(dtype=torch.float32) if args.decode_fp32 else ModelShape()
     g = args.decode_grid
     prompt = [int(x) for x in torch.randint(0, shape.vocab, (16,), generator=torch.Generator().manual_seed(7))]
-    dec = Decoder(shape, batch=args.decode_batch, grid=(g, g), prompt_len=16, seed=2025)
+    graphs = not args.decode_eager
+    dec = Decoder(shape, batch=args.decode_batch, grid=(g, g), prompt_len=16, seed=2025, graphs=graphs)
     # warm-up: a small grid with the same weights (cuBLAS plans, library set-up)
     Decoder(shape, batch=args.decode_batch, grid=(4, 4), prompt_len=16, seed=2025,
             target=dec.target_w).generate(prompt)
     out, st = dec.generate(prompt)
     n = g * g
     t0 = time.perf_counter()
-    ref, margins = greedy_decode(shape, dec.target_w, prompt, n, batch=args.decode_batch, return_margins=True)
+    ref, margins = greedy_decode(shape, dec.target_w, prompt, n, batch=args.decode_batch, return_margins=True,
+                                 graphs=graphs)
     torch.cuda.synchronize()
     t_van = time.perf_counter() - t0
     same = sum(1 for b in range(args.decode_batch) for x, y in zip(out[b], ref[b]) if x == y)
@@ -428,7 +430,8 @@ def run_decode(args):
                                    f"11008, vocab 65536) + one-layer EAGLE-style draft head, {g}x{g} image tokens "
                                    f"after a 16-token prompt, ADT-Tree controller (Anole bounds), greedy",
                        "batch": args.decode_batch,
-                       "dense_dtype": "fp32" if args.decode_fp32 else "bf16"},
+                       "dense_dtype": "fp32" if args.decode_fp32 else "bf16",
+                       "launch": "CUDA graph per tree size" if graphs else "eager"},
             "tau": st.tau, "accepted_draft_tokens": st.accepted, "verify_steps": st.steps,
             "mean_depth": st.mean_depth, "seconds": st.seconds,
             "vanilla_greedy_tokens_per_s": args.decode_batch * n / t_van,
@@ -457,6 +460,7 @@ def main():
     ap.add_argument("--decode-batch", type=int, default=1)
     ap.add_argument("--decode-grid", type=int, default=48)
     ap.add_argument("--decode-fp32", action="store_true", help="fp32 weights and residual stream in the harness")
+    ap.add_argument("--decode-eager", action="store_true", help="no CUDA graphs in the decode loop")
     args = ap.parse_args()
     if args.decode:
         run_decode(args)

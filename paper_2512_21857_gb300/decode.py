@@ -118,6 +118,8 @@ class TreeModel:
         self.ws = B.zeroed_workspace(B.adt_tree_attn_workspace_size(batch, s.heads, s.head_dim, max_nodes, lmax),
                                      device)
         self.device = device
+        self.graphs_enabled = False
+        self._graphs = {}
 
     def forward(self, x, pos, parents, node_offsets, kv_len, batch, image=None):
         """x [N, hidden] (bf16) for the nodes of `batch` trees (of image
@@ -148,6 +150,32 @@ class TreeModel:
             gu = h @ lw["wgu"]
             x = x + (torch.nn.functional.silu(gu[:, : s.ffn].float()) * gu[:, s.ffn:].float()).to(x.dtype) @ lw["wd"]
         return x, k_tree, v_tree
+
+    def run(self, x, pos, parents, node_offsets, kv_len, batch, image=None):
+        """forward() through a CUDA graph captured once per (nodes, batch,
+        image): the stack's few hundred launches replay without host work.
+        The outputs are the graph's own buffers, rewritten by the next replay
+        of the same shape: copy what must outlive it."""
+        if not self.graphs_enabled:
+            return self.forward(x, pos, parents, node_offsets, kv_len, batch, image)
+        key = (x.shape[0], batch, image)
+        g = self._graphs.get(key)
+        if g is None:
+            ins = [t.clone() for t in (x, pos, parents, node_offsets, kv_len)]
+            side = torch.cuda.Stream()
+            side.wait_stream(torch.cuda.current_stream())
+            with torch.cuda.stream(side):
+                self.forward(*ins, batch, image)  # warm-up outside the capture
+            torch.cuda.current_stream().wait_stream(side)
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph):
+                outs = self.forward(*ins, batch, image)
+            g = self._graphs[key] = (graph, ins, outs)
+        graph, ins, outs = g
+        for dst, src in zip(ins, (x, pos, parents, node_offsets, kv_len)):
+            dst.copy_(src)
+        graph.replay()
+        return outs
 
     def commit(self, k_tree, v_tree, kv_len, kv_len_out, node_offsets, path, max_path, accept_len, batch):
         B.adt_kv_compact(self.k_cache, self.v_cache, kv_len, kv_len_out, k_tree, v_tree, node_offsets, path,
@@ -193,7 +221,7 @@ class Decoder:
     tokens after a prompt (the same prompt for every image)."""
 
     def __init__(self, shape: ModelShape, *, batch=1, grid=(48, 48), prompt_len=16, seed=2025, device="cuda",
-                 max_nodes=64, ctrl_params=None, draft_equals_target=False, target=None):
+                 max_nodes=64, ctrl_params=None, draft_equals_target=False, target=None, graphs=False):
         s = self.s = shape
         self.batch, self.grid, self.prompt_len = batch, grid, prompt_len
         self.device = device
@@ -215,6 +243,7 @@ class Decoder:
             dw = DecoderWeights(s, 1, seed + 1, device, lm=False, draft_fc=True)
         self.draft_w = dw
         self.draft = TreeModel(s, dw, batch, self.lmax, 256, device)
+        self.target.graphs_enabled = self.draft.graphs_enabled = graphs
         self.ctrl_params = dict(ctrl_params or {})
         self.ctrl_params.setdefault("d_lo", 1)
         self.ctrl_params.setdefault("d_hi", 9)
@@ -250,7 +279,7 @@ class Decoder:
         offs = self._i32([b * n for b in range(Bn + 1)])
         zero = self._i32([0] * Bn)
         pos = torch.arange(n, device=dev, dtype=torch.int32).repeat(Bn)
-        h, kt, vt = self.target.forward(self._embed(tok), pos, par, offs, zero, Bn)
+        h, kt, vt = self.target.run(self._embed(tok), pos, par, offs, zero, Bn)
         path = torch.arange(n, dtype=torch.int32, device=dev).repeat(Bn, 1).contiguous()
         alen = self._i32([n - 1] * Bn)
         kv_out = torch.empty(Bn, dtype=torch.int32, device=dev)
@@ -261,7 +290,8 @@ class Decoder:
         for b in range(Bn):
             # the draft catches up on prompt[:-1]: parent features f_{t-1} (zeros for t = 0)
             pf = torch.cat([zf[None], feats[b, :-1]], 0)
-            state.append(dict(kv=n, dkv=0, root=int(prompt[-1]), root_pf=feats[b, -1], catch_tok=list(prompt[:-1]),
+            state.append(dict(kv=n, dkv=0, root=int(prompt[-1]), root_pf=feats[b, -1].clone(),
+                              catch_tok=list(prompt[:-1]),
                               catch_pf=pf, pos=0))
         return state
 
@@ -293,7 +323,7 @@ class Decoder:
             n = tok.numel()
             x = torch.cat([self._embed(tok), pf], 1) @ self.draft_w.fc
             offs = self._i32([0, n])
-            h, kt, vt = self.draft.forward(x, st["dkv"] + dep, par, offs, dkv, 1, image=b)
+            h, kt, vt = self.draft.run(x, st["dkv"] + dep, par, offs, dkv, 1, image=b)
             logits = self._logits(h[front]).contiguous()
             F = front.numel()
             keep = torch.empty(width, dtype=torch.int32, device=dev)
@@ -352,7 +382,7 @@ class Decoder:
         par = torch.cat([t["parents"] for t in trees])
         kv = self._i32([st["kv"] for st in state])
         pos = torch.cat([t["depth"] + st["kv"] for t, st in zip(trees, state)])
-        h, kt, vt = self.target.forward(self._embed(tok), pos, par, offs, kv, Bn)
+        h, kt, vt = self.target.run(self._embed(tok), pos, par, offs, kv, Bn)
         logits = self._logits(h).contiguous()
         max_path = max(d for d, _ in dk) + 1
         path = torch.full((Bn, max_path), -1, dtype=torch.int32, device=dev)
@@ -380,7 +410,7 @@ class Decoder:
             st["catch_tok"] = toks
             st["catch_pf"] = torch.cat([st["root_pf"][None], h[idx[:-1]]], 0)
             st["root"] = bonus_h[b]
-            st["root_pf"] = h[idx[-1]]
+            st["root_pf"] = h[idx[-1]].clone()
             st["kv"] += a + 1
             st["pos"] += len(new)
         return emitted, dk, alen_h
@@ -414,7 +444,7 @@ class Decoder:
 
 
 def greedy_decode(shape: ModelShape, weights: DecoderWeights, prompt, n_tokens, device="cuda", batch=1,
-                  return_margins=False):
+                  return_margins=False, graphs=False):
     """Vanilla greedy decoding with the same target: one node per step (a
     tree of its root alone).  Returns the tokens (and, with return_margins,
     the top-1 minus top-2 logit gap of every decision over the standard
@@ -422,6 +452,7 @@ def greedy_decode(shape: ModelShape, weights: DecoderWeights, prompt, n_tokens, 
     if not 2 <= len(prompt) <= 257:
         raise ValueError("prompt of 2 .. 257 tokens (the prefill is one tree)")
     model = TreeModel(shape, weights, batch, len(prompt) + n_tokens + 16, len(prompt) - 1, device)
+    model.graphs_enabled = graphs
     dev = device
     P = len(prompt)
     n = P - 1
@@ -431,7 +462,7 @@ def greedy_decode(shape: ModelShape, weights: DecoderWeights, prompt, n_tokens, 
     offs = torch.tensor([b * n for b in range(batch + 1)], **i32)
     kv = torch.zeros(batch, **i32)
     pos = torch.arange(n, device=dev, dtype=torch.int32).repeat(batch)
-    _, kt, vt = model.forward(weights.embed[tok.long()], pos, par, offs, kv, batch)
+    _, kt, vt = model.run(weights.embed[tok.long()], pos, par, offs, kv, batch)
     path = torch.arange(n, **i32).repeat(batch, 1).contiguous()
     kv_out = torch.empty(batch, **i32)
     model.commit(kt, vt, kv, kv_out, offs, path, n, torch.full((batch,), n - 1, **i32), batch)
@@ -443,7 +474,7 @@ def greedy_decode(shape: ModelShape, weights: DecoderWeights, prompt, n_tokens, 
     zpath = torch.zeros((batch, 1), **i32)
     zlen = torch.zeros(batch, **i32)
     for _ in range(n_tokens):
-        h, kt, vt = model.forward(weights.embed[root.long()], kv, rootpar, one, kv, batch)
+        h, kt, vt = model.run(weights.embed[root.long()], kv, rootpar, one, kv, batch)
         logits = lm_logits(weights, h, shape.eps)
         top2 = torch.topk(logits, 2, dim=-1)
         nxt = top2.indices[:, 0].to(torch.int32)

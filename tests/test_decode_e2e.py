@@ -42,12 +42,12 @@ SMALL = ModelShape(layers=2, hidden=256, heads=2, kv_heads=2, head_dim=128, ffn=
                   lm_std=1.0)
 
 
-@pytest.mark.parametrize("batch", [1, 2])
-def test_adt_decode_equals_greedy(batch):
-    dec = Decoder(SMALL, batch=batch, grid=(8, 8), prompt_len=8, seed=7, max_nodes=64)
+@pytest.mark.parametrize("batch,graphs", [(1, False), (2, False), (2, True)])
+def test_adt_decode_equals_greedy(batch, graphs):
+    dec = Decoder(SMALL, batch=batch, grid=(8, 8), prompt_len=8, seed=7, max_nodes=64, graphs=graphs)
     prompt = _prompt(SMALL.vocab, 8, 1)
     out, stats = dec.generate(prompt)
-    ref, margins = greedy_decode(SMALL, dec.target_w, prompt, 64, batch=batch, return_margins=True)
+    ref, margins = greedy_decode(SMALL, dec.target_w, prompt, 64, batch=batch, return_margins=True, graphs=graphs)
     for b in range(batch):
         assert len(out[b]) == 64
         n = _compare(out[b], ref[b], margins[b])
