@@ -40,6 +40,12 @@ WORKLOADS = {
     "c1": dict(name="single verify step: 1 layer, 8 heads x 64, KV 512, 26-node tree (depth 4, width 4), "
                     "vocab 16384, batch 1",
                layers=1, H=8, Hkv=8, D=64, V=16384, kv_len=[512], depth=[4], width=[4], max_nodes=26),
+    # prefix lengths ~ U{600..2400}, depths ~ U{2..10}, widths ~ U{1..8} (numpy default_rng(20251221), in
+    # that order): one batched step of the adjacency-adaptive sweep, each image's tree its own shape
+    "c4": dict(name="adjacency-adaptive ragged batch: 8 images at the 7B shape (32 layers, 32 heads x 128, "
+                    "vocab 65536), KV 600-2400, per-image depth 2-10 and width 1-8, trees of up to 64 nodes",
+               layers=32, H=32, Hkv=32, D=128, V=65536, kv_len=[751, 1596, 1444, 640, 1427, 1245, 2352, 1248],
+               depth=[4, 7, 8, 7, 6, 6, 7, 6], width=[6, 8, 4, 2, 2, 1, 6, 4], max_nodes=64),
 }
 
 # DRAM bytes (read + write) of one tree_attn launch at the 7B shape, from one
@@ -314,14 +320,15 @@ class OracleSample:
     full rerank and greedy acceptance walk, and the KV commit of one layer.
     Inputs are drawn once; run() times only the oracle calls."""
 
-    def __init__(self, wl, seed, heads, layers_sampled, rows_sampled):
+    def __init__(self, wl, seed, heads, layers_sampled, rows_sampled, image=0):
         import numpy as np
 
         from paper_2512_21857_gb300 import synth
 
         self.wl = wl
-        H, Hkv, D, V, L = wl["H"], wl["Hkv"], wl["D"], wl["V"], wl["kv_len"][0]
-        k, depth, nmax = wl["width"][0], wl["depth"][0], wl["max_nodes"]
+        self.image = image
+        H, Hkv, D, V, L = wl["H"], wl["Hkv"], wl["D"], wl["V"], wl["kv_len"][image]
+        k, depth, nmax = wl["width"][image], wl["depth"][image], wl["max_nodes"]
         self.n = n = min(nmax, k + (depth - 1) * k * k + 1)
         self.hs = hs = max(1, min(heads, H))
         self.layers_sampled = layers_sampled
@@ -334,6 +341,7 @@ class OracleSample:
         self.vc = synth.bf16_normal((1, hs, L, D), seed, "vc").double().numpy()
         self.kt = synth.bf16_normal((n, hs, D), seed, "kt").double().numpy()
         self.vt = synth.bf16_normal((n, hs, D), seed, "vt").double().numpy()
+        self.rows_sampled = rows_sampled = min(rows_sampled, self.total_rows)
         self.rows = synth.f32_normal((rows_sampled, V), seed, "rows")
         self.target = synth.f32_normal((n, V), seed, "target")
         C = k + (depth - 1) * k * k
@@ -353,7 +361,7 @@ class OracleSample:
         import oracle
 
         wl = self.wl
-        L, D, n, k = wl["kv_len"][0], wl["D"], self.n, wl["width"][0]
+        L, D, n, k = wl["kv_len"][self.image], wl["D"], self.n, wl["width"][self.image]
         t = time.perf_counter()
         for _ in range(self.layers_sampled):
             oracle.tree_attention(self.q, self.kc, self.vc, [L], self.kt, self.vt, self.tb.parents, [0, n],
@@ -386,9 +394,13 @@ def cpu_sample_subprocess(wl_key, heads, layers_sampled, rows_sampled, reps):
 
 def cpu_sample_main(args):
     wl = WORKLOADS[args.cpu_sample]
-    sample = OracleSample(wl, 7, args.cpu_heads, args.cpu_layers, args.cpu_rows)
-    times = [sample.run() for _ in range(args.cpu_reps)]
-    print(json.dumps({"sec_per_step": times, "desc": sample.desc}))
+    samples = [OracleSample(wl, 7 + b, args.cpu_heads, args.cpu_layers, args.cpu_rows, image=b)
+               for b in range(len(wl["kv_len"]))]
+    times = [sum(smp.run() for smp in samples) for _ in range(args.cpu_reps)]
+    desc = samples[0].desc
+    if len(samples) > 1:
+        desc = f"per image of the {len(samples)}, summed: " + desc
+    print(json.dumps({"sec_per_step": times, "desc": desc}))
 
 
 # ------------------------------------------------------------------ main
@@ -473,11 +485,15 @@ def main():
     wl = WORKLOADS[args.workload]
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
-    config = {"workload": wl["name"], "batch": len(wl["kv_len"]), "kv_len": wl["kv_len"][0],
-              "tree_nodes": wl["max_nodes"], "depth": wl["depth"][0], "width": wl["width"][0], "vocab": wl["V"],
+    one = len(wl["kv_len"]) == 1
+    config = {"workload": wl["name"], "batch": len(wl["kv_len"]), "kv_len": wl["kv_len"][0] if one else wl["kv_len"],
+              "tree_nodes": wl["max_nodes"], "depth": wl["depth"][0] if one else wl["depth"],
+              "width": wl["width"][0] if one else wl["width"], "vocab": wl["V"],
               "layers": wl["layers"], "heads": wl["H"], "head_dim": wl["D"], "accept_mode": args.mode,
               "l2": "inputs larger than L2: every layer reads its own 39 MB KV cache slice (1.3 GB per step)"
-                    if args.workload == "7b" else "per-step inputs rotate through distinct layer buffers",
+                    if args.workload == "7b" else
+                    "inputs larger than L2: every layer reads its own KV cache slices (188 MB per layer, 6.0 GB "
+                    "per step)" if args.workload == "c4" else "per-step inputs rotate through distinct layer buffers",
               "parallelism": f"replicas x{world}"}
     metric = "tree-verify steps/s"
 
@@ -516,7 +532,10 @@ def main():
     e2e_value = world * 1e3 / r["e2e_ms"]
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
-        res = cpu_sample_subprocess(args.workload, wl["H"], 1, 41, 5)
+        if one:
+            res = cpu_sample_subprocess(args.workload, wl["H"], 1, 41, 5)
+        else:  # a bounded sample: 4 heads of one layer per image
+            res = cpu_sample_subprocess(args.workload, 4, 1, 8, 3)
         sec = statistics.median(res["sec_per_step"])
         cpu = {"value": 1.0 / sec, "unit": "steps/s", "cores": 1, "kind": "oracle", "sample": res["desc"]}
     line = {
