@@ -5,9 +5,11 @@ tree) and the HBM roofline of the attention kernel.
 One step = 6 draft-layer expansions (width 8) over 65536-entry draft rows,
 the top-63 rerank, tree attention over all 32 layers (32 heads x 128, prefix
 2400), the acceptance walk and the KV commit of the accepted path: every row
-of the hot path, as one sequence of library launches (three CUDA graphs).
+of the hot path, as one CUDA graph of library launches.  The attention
+kernel's time per launch (the roofline) comes from a second timed region in
+the same run: the 32 attention layers alone, back to back as in the step.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 7b|llamagen|c1]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 7b|llamagen|c1|c4]
                   [--mode greedy|spec_det] [--impl adt|reference]
 
 Prints one JSON line.  With torchrun (N > 1) every rank runs an independent
@@ -167,35 +169,29 @@ def run_gpu(args, wl, rank, world):
     torch.cuda.synchronize()
     if B.adt_get_device_error(stream) != 0:
         raise RuntimeError("device error flag set during the eager pass")
-    graphs = [torch.cuda.CUDAGraph() for _ in range(3)]
+    # The step is one CUDA graph (its kernels chained by programmatic
+    # dependent launch, no host work between them).  The attention layers
+    # are also captured alone, back to back as inside the step, to time the
+    # attention kernel for the roofline in a second timed region.
+    step_graph = torch.cuda.CUDAGraph()
+    attn_graph = torch.cuda.CUDAGraph()
     with torch.cuda.stream(stream):
-        with torch.cuda.graph(graphs[0], stream=stream):
-            step.launch_draft(stream)
-        with torch.cuda.graph(graphs[1], stream=stream):
+        with torch.cuda.graph(step_graph, stream=stream):
+            step.launch(stream)
+        with torch.cuda.graph(attn_graph, stream=stream):
             for layer in range(shape.layers):
                 step.launch_attention(layer, stream)
-        with torch.cuda.graph(graphs[2], stream=stream):
-            step.launch_verify(stream)
     torch.cuda.synchronize()
-
-    def one_step(ev_a=None, ev_b=None):
-        graphs[0].replay()
-        if ev_a is not None:
-            ev_a.record(stream)
-        graphs[1].replay()
-        if ev_b is not None:
-            ev_b.record(stream)
-        graphs[2].replay()
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
-            one_step()
+            step_graph.replay()
+            attn_graph.replay()
     torch.cuda.synchronize()
 
     K = args.steps
-    ev_a = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
-    ev_b = [torch.cuda.Event(enable_timing=True) for _ in range(K)]
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ea0, ea1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     sampler = ClockSampler(local)
     sampler.start()
     time.sleep(0.4)
@@ -205,16 +201,20 @@ def run_gpu(args, wl, rank, world):
     t0 = time.time()
     with torch.cuda.stream(stream):
         ev0.record(stream)
-        for i in range(K):
-            one_step(ev_a[i], ev_b[i])
+        for _ in range(K):
+            step_graph.replay()
         ev1.record(stream)
+        ea0.record(stream)
+        for _ in range(K):
+            attn_graph.replay()
+        ea1.record(stream)
     torch.cuda.synchronize()
     t1 = time.time()
     if world > 1:
         torch.distributed.barrier()
     clocks = sampler.stop(t0, t1)
     step_ms = ev0.elapsed_time(ev1) / K
-    attn_ms = sum(a.elapsed_time(b) for a, b in zip(ev_a, ev_b)) / (K * shape.layers)
+    attn_ms = ea0.elapsed_time(ea1) / (K * shape.layers)
     errbits = B.adt_get_device_error(stream)
     if errbits:
         raise RuntimeError(f"device error bits {errbits:#x} during the timed steps")
@@ -236,18 +236,13 @@ def run_gpu(args, wl, rank, world):
                 a.copy_(b_)
         else:
             dst.copy_(src)
-    graphs1 = [torch.cuda.CUDAGraph() for _ in range(3)]
+    step_graph1 = torch.cuda.CUDAGraph()
     with torch.cuda.stream(stream):
-        with torch.cuda.graph(graphs1[0], stream=stream):
-            step.launch_draft(stream)
-        with torch.cuda.graph(graphs1[1], stream=stream):
-            for layer in range(shape.layers):
-                step.launch_attention(layer, stream)
-        with torch.cuda.graph(graphs1[2], stream=stream):
-            step.launch_verify(stream)
+        with torch.cuda.graph(step_graph1, stream=stream):
+            step.launch(stream)
     step.use_slot(0)
     torch.cuda.synchronize()
-    slot_graphs = [graphs, graphs1]
+    slot_graphs = [step_graph, step_graph1]
     slot_inputs = []
     for i in range(2):
         step.use_slot(i)
@@ -273,8 +268,7 @@ def run_gpu(args, wl, rank, world):
             copied[sl].record(copy_stream)
         stream.wait_event(copied[sl])
         with torch.cuda.stream(stream):
-            for gr in slot_graphs[sl]:
-                gr.replay()
+            slot_graphs[sl].replay()
             consumed[sl].record(stream)
             for h, d in zip(host_out[sl], outputs):
                 h.copy_(d, non_blocking=True)
@@ -307,7 +301,7 @@ def run_gpu(args, wl, rank, world):
     sha = attn_source_sha()
     traffic = NCU_TRAFFIC.get(sha) if args.workload == "7b" else None
     return dict(step_ms=step_ms, attn_ms=attn_ms, clocks=clocks, e2e_ms=e2e_ms, h2d=h2d, d2h=d2h,
-                launches=K * step.kernel_launches_per_step(), achieved=achieved, peak=peak, peak_kind=peak_kind,
+                launches=K * (step.kernel_launches_per_step() + shape.layers), achieved=achieved, peak=peak, peak_kind=peak_kind,
                 traffic=traffic, attn_bytes=ab["attention_per_layer"], step_bytes=ab["attention"], sha=sha)
 
 
