@@ -57,6 +57,16 @@ constexpr unsigned kFullMask = 0xffffffffu;
 // stream has completed and its memory is visible (immediate when this launch
 // does not overlap one), then let the next kernel begin launching.  Called
 // before the kernel's first global-memory access.
+// Atomic add at device scope with acquire-release order: writes made
+// visible to the calling thread before it (e.g. through a block barrier)
+// are published with it, and what other threads published with their own
+// add is visible after it.  Returns the old value.
+__device__ __forceinline__ unsigned atomic_add_acq_rel_gpu(unsigned* addr, unsigned v) {
+  unsigned old;
+  asm volatile("atom.add.acq_rel.gpu.u32 %0, [%1], %2;\n" : "=r"(old) : "l"(addr), "r"(v) : "memory");
+  return old;
+}
+
 __device__ __forceinline__ void pdl_wait_then_release() {
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
   asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");

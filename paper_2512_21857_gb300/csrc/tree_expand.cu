@@ -248,6 +248,11 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
   const float* row_u = p.logits_u ? p.logits_u + static_cast<int64_t>(r) * p.ld : nullptr;
   float* vals_u = vals + min(per, kTile);  // used only with guidance
 
+  // The row's frontier score and id, read now by the threads that write the
+  // children at the end: the loads' latency hides behind the passes.
+  const bool writer = rank == 0 && tid < K;
+  const float f_score = writer ? p.fscore[r] : 0.f;
+  const int32_t f_id = writer ? (p.fid ? p.fid[r] : r) : 0;
   for (int i = tid; i < kMaxK; i += kThreads) ctl[i] = 0ull;
   if (tid == 0) {
     s_cnt = 0u;
@@ -398,23 +403,36 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
   __syncthreads();
   rank_select(cl_keys, C * K, K, rowl);
   __syncthreads();
-  if (tid < K) {
+  if (writer) {
     const uint64_t key = rowl[tid];
     const double lp = static_cast<double>(adt::select_key_value(key)) - s_lse;
-    const float score = static_cast<float>(static_cast<double>(p.fscore[r]) + lp);
+    const float score = static_cast<float>(static_cast<double>(f_score) + lp);
     const int64_t c = static_cast<int64_t>(r) * K + tid;
     p.ctok[c] = static_cast<int32_t>(adt::select_key_index(key));
     if (p.clogp) p.clogp[c] = static_cast<float>(lp);
     p.cscore[c] = score;
-    p.cpar[c] = p.fid ? p.fid[r] : r;
-    p.cross_keys[c] = adt::select_key(score, static_cast<uint32_t>(c));
+    p.cpar[c] = f_id;
+    if (p.F == 1) {
+      // One row: its children are already in score order (the score grows
+      // with the log-probability; ties keep the lower index, as the
+      // cross-row ranking would), so the next frontier is their first k_keep.
+      if (tid < p.k_keep) {
+        p.keep[tid] = static_cast<int32_t>(c);
+        if (p.nscore) p.nscore[tid] = score;
+        if (p.nid) p.nid[tid] = p.id_base + static_cast<int32_t>(c);
+      }
+    } else {
+      p.cross_keys[c] = adt::select_key(score, static_cast<uint32_t>(c));
+    }
   }
-  __threadfence();
+  if (p.F == 1) return;
+  // The row's cross keys are written (CTA order); the ticket's release
+  // publishes them at device scope and its acquire, in the last row, makes
+  // every row's keys visible.
   __syncthreads();
-  if (tid == 0) s_last = atomicAdd(p.all_ticket, 1u) == static_cast<unsigned>(p.F - 1);
+  if (tid == 0) s_last = adt::atomic_add_acq_rel_gpu(p.all_ticket, 1u) == static_cast<unsigned>(p.F - 1);
   __syncthreads();
   if (!s_last) return;
-  __threadfence();
 
   // ---- last row: next frontier across all rows.
   const int nc = p.F * K;
