@@ -929,15 +929,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   }
-  __threadfence();
   sm100::cluster_wait_acquire();  // pairs with the prologue's arrive (a cluster of one CTA here)
   __syncthreads();
   sm100::tc_fence_after();
   if (warp == 0) sm100::tmem_dealloc(tmem, kTmemCols);
-  if (tid == 0) s_last = atomicAdd(p.tickets + bh, 1u) == static_cast<unsigned>(S - 1);
+  // The ticket's release publishes this split's partials (ordered before it
+  // by the barrier); its acquire, in the last split, makes all of them visible.
+  if (tid == 0) s_last = adt::atomic_add_acq_rel_gpu(p.tickets + bh, 1u) == static_cast<unsigned>(S - 1);
   __syncthreads();
   if (!s_last) return;
-  __threadfence();
   const float* po_bh = p.part_o + bh * S * kMaxNodes * D;
   const float2* pml_bh = p.part_ml + bh * S * kMaxNodes;
   float* wsm = reinterpret_cast<float*>(sStage);  // [64][S]

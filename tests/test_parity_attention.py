@@ -22,6 +22,8 @@ CASES = [
     ([33, 7, 1, 64], [63, 64, 65, 0], 4, 4, 128),  # ragged batch, tile edges, empty prefix
     ([12, 5], [700, 1], 8, 2, 128),       # grouped kv heads
     ([1], [300], 4, 4, 64),               # single node = ordinary decode attention
+    ([40], [2400], 2, 2, 128),            # few heads, long prefix: 20 splits merge through the workspace
+    ([64, 9], [4000, 3000], 2, 1, 64),    # the same with grouped heads, two trees
 ]
 
 
