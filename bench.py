@@ -62,6 +62,24 @@ def log(*a):
     print(*a, file=sys.stderr, flush=True)
 
 
+def max_over_ranks(x: float, world: int) -> float:
+    """The largest of every rank's x (the slowest replica sets the job's
+    time); x itself with one rank."""
+    if world <= 1:
+        return x
+    import torch
+    dev = "cuda" if torch.distributed.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(ms_per_step: float, world: int) -> float:
+    """Whole-job steps/s: every rank verifies its own replica's step (weak
+    scaling), in the slowest rank's time."""
+    return world * 1e3 / ms_per_step
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -218,10 +236,7 @@ def run_gpu(args, wl, rank, world):
     errbits = B.adt_get_device_error(stream)
     if errbits:
         raise RuntimeError(f"device error bits {errbits:#x} during the timed steps")
-    if world > 1:
-        t = torch.tensor([step_ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        step_ms = float(t.item())
+    step_ms = max_over_ranks(step_ms, world)
 
     # End to end through the public API: every step copies its inputs from
     # pinned host memory into one of two input slots and reads its result
@@ -290,10 +305,7 @@ def run_gpu(args, wl, rank, world):
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1) / K2
-    if world > 1:
-        t = torch.tensor([e2e_ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = max_over_ranks(e2e_ms, world)
 
     ab = step.algorithmic_bytes()
     peak, peak_kind = measured_peaks()
@@ -522,8 +534,8 @@ def main():
             import torch
             torch.distributed.destroy_process_group()
         return
-    value = world * 1e3 / r["step_ms"]
-    e2e_value = world * 1e3 / r["e2e_ms"]
+    value = job_throughput(r["step_ms"], world)
+    e2e_value = job_throughput(r["e2e_ms"], world)
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         if one:
