@@ -53,8 +53,8 @@ WORKLOADS = {
 # DRAM bytes (read + write) of one tree_attn launch at the 7B shape, from one
 # ncu capture; valid only for the kernel source with this SHA-256 prefix.
 NCU_TRAFFIC = {
-    # dram__bytes_read.sum + dram__bytes_write.sum = 41,492,992 + 0
-    "22ecb2dbc47cd30e": 41492992,
+    # dram__bytes_read.sum + dram__bytes_write.sum = 41,492,736 + 2,816
+    "0f73e9a989852d49": 41495552,
 }
 
 
