@@ -326,7 +326,7 @@ class OracleSample:
     full rerank and greedy acceptance walk, and the KV commit of one layer.
     Inputs are drawn once; run() times only the oracle calls."""
 
-    def __init__(self, wl, seed, heads, layers_sampled, rows_sampled, image=0):
+    def __init__(self, wl, seed, heads, layers_sampled, rows_sampled, image=0, nodes_sampled=0):
         import numpy as np
 
         from paper_2512_21857_gb300 import synth
@@ -336,6 +336,9 @@ class OracleSample:
         H, Hkv, D, V, L = wl["H"], wl["Hkv"], wl["D"], wl["V"], wl["kv_len"][image]
         k, depth, nmax = wl["width"][image], wl["depth"][image], wl["max_nodes"]
         self.n = n = min(nmax, k + (depth - 1) * k * k + 1)
+        # attention over the first nq nodes (parents precede children, so a
+        # prefix of the node list is itself a tree), extrapolated to n
+        self.nq = nq = n if nodes_sampled <= 0 else max(1, min(n, nodes_sampled))
         self.hs = hs = max(1, min(heads, H))
         self.layers_sampled = layers_sampled
         self.rows_sampled = rows_sampled
@@ -357,7 +360,8 @@ class OracleSample:
         self.kc16 = np.zeros((1, 1, Hkv, L + nmax, D), np.int16)
         self.kt16 = np.zeros((1, n, Hkv, D), np.int16)
         self.desc = (f"oracle (numpy fp64, 1 thread) on {hs} of {H} heads x {layers_sampled} of {wl['layers']} "
-                     f"layers of attention, {rows_sampled} of {self.total_rows} draft rows of expansion, full "
+                     f"layers of attention" + (f" for {nq} of {n} tree nodes" if nq < n else "") +
+                     f", {rows_sampled} of {self.total_rows} draft rows of expansion, full "
                      f"rerank and greedy walk, 1 of {wl['layers']} layers of KV commit; extrapolated linearly "
                      f"to one full step")
 
@@ -369,10 +373,12 @@ class OracleSample:
         wl = self.wl
         L, D, n, k = wl["kv_len"][self.image], wl["D"], self.n, wl["width"][self.image]
         t = time.perf_counter()
+        nq = self.nq
         for _ in range(self.layers_sampled):
-            oracle.tree_attention(self.q, self.kc, self.vc, [L], self.kt, self.vt, self.tb.parents, [0, n],
-                                  1.0 / math.sqrt(D))
-        t_attn = (time.perf_counter() - t) / self.layers_sampled * wl["layers"] * (wl["H"] / self.hs)
+            oracle.tree_attention(self.q[:nq], self.kc, self.vc, [L], self.kt[:nq], self.vt[:nq],
+                                  self.tb.parents[:nq], [0, nq], 1.0 / math.sqrt(D))
+        t_attn = ((time.perf_counter() - t) / self.layers_sampled * wl["layers"] * (wl["H"] / self.hs)
+                  * (n / nq))
         t = time.perf_counter()
         oracle.tree_expand(self.rows, np.zeros(self.rows_sampled, np.float32), k, k)
         t_exp = (time.perf_counter() - t) / self.rows_sampled * self.total_rows
@@ -386,12 +392,13 @@ class OracleSample:
         return t_attn + t_exp + t_acc + t_cmp
 
 
-def cpu_sample_subprocess(wl_key, heads, layers_sampled, rows_sampled, reps):
+def cpu_sample_subprocess(wl_key, heads, layers_sampled, rows_sampled, reps, nodes=0):
     """Runs oracle samples in a fresh single-threaded process."""
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
                CUDA_VISIBLE_DEVICES="")
     cmd = [sys.executable, os.path.abspath(__file__), "--cpu-sample", wl_key, "--cpu-heads", str(heads),
-           "--cpu-layers", str(layers_sampled), "--cpu-rows", str(rows_sampled), "--cpu-reps", str(reps)]
+           "--cpu-layers", str(layers_sampled), "--cpu-rows", str(rows_sampled), "--cpu-reps", str(reps),
+           "--cpu-nodes", str(nodes)]
     out = subprocess.run(cmd, capture_output=True, text=True, env=env, timeout=1800)
     if out.returncode != 0:
         raise RuntimeError(out.stderr[-2000:])
@@ -400,7 +407,8 @@ def cpu_sample_subprocess(wl_key, heads, layers_sampled, rows_sampled, reps):
 
 def cpu_sample_main(args):
     wl = WORKLOADS[args.cpu_sample]
-    samples = [OracleSample(wl, 7 + b, args.cpu_heads, args.cpu_layers, args.cpu_rows, image=b)
+    samples = [OracleSample(wl, 7 + b, args.cpu_heads, args.cpu_layers, args.cpu_rows, image=b,
+                            nodes_sampled=args.cpu_nodes)
                for b in range(len(wl["kv_len"]))]
     times = [sum(smp.run() for smp in samples) for _ in range(args.cpu_reps)]
     desc = samples[0].desc
@@ -474,6 +482,7 @@ def main():
     ap.add_argument("--cpu-layers", type=int, default=1)
     ap.add_argument("--cpu-rows", type=int, default=1)
     ap.add_argument("--cpu-reps", type=int, default=1)
+    ap.add_argument("--cpu-nodes", type=int, default=0)
     ap.add_argument("--decode", action="store_true", help="the end-to-end synthetic decode loop instead")
     ap.add_argument("--decode-batch", type=int, default=1)
     ap.add_argument("--decode-grid", type=int, default=48)
@@ -511,7 +520,12 @@ def main():
         if rank != 0:
             return
         t_run = time.time()
-        res = cpu_sample_subprocess(args.workload, 1, 1, 1, args.warmup + args.steps)
+        # Each step's sample shrinks with the step count so that the run stays
+        # within a few minutes: past 1000 steps, attention covers a prefix of
+        # the tree's nodes in proportion.
+        n_steps = args.warmup + args.steps
+        nodes = 0 if n_steps <= 1000 else max(4, (64 * 1000) // n_steps)
+        res = cpu_sample_subprocess(args.workload, 1, 1, 1, n_steps, nodes)
         samples = res["sec_per_step"][args.warmup:]
         sec = statistics.mean(samples)
         value = 1.0 / sec
