@@ -52,9 +52,10 @@ WORKLOADS = {
 
 # DRAM bytes (read + write) of one tree_attn launch at the 7B shape, from one
 # ncu capture; valid only for the kernel source with this SHA-256 prefix.
+HOST_MARKER = b"// ---------------------------------------------------------------- host side"
 NCU_TRAFFIC = {
     # dram__bytes_read.sum + dram__bytes_write.sum = 41,492,736 + 2,816
-    "0f73e9a989852d49": 41495552,
+    "c9b603a818f5df14": 41495552,
 }
 
 
@@ -90,8 +91,12 @@ def measured_peaks():
 
 
 def attn_source_sha():
+    """SHA-256 prefix of the attention kernel's device code: tree_attn.cu up to
+    its host-side section (host-only edits do not change the kernel)."""
     with open(os.path.join(ROOT, "paper_2512_21857_gb300", "csrc", "tree_attn.cu"), "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+        src = f.read()
+    cut = src.find(HOST_MARKER)
+    return hashlib.sha256(src if cut < 0 else src[:cut]).hexdigest()[:16]
 
 
 # ------------------------------------------------------------------ clocks

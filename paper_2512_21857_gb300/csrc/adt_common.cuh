@@ -6,8 +6,19 @@
 #include <stdint.h>
 
 #include "adt.h"
+#include <nvtx3/nvToolsExt.h>
 
 namespace adt {
+
+// An NVTX range named after the library call, for profilers' timelines
+// (header-only NVTX: without a tool attached a push and a pop cost a few
+// nanoseconds).
+struct TraceRange {
+  explicit TraceRange(const char* name) { nvtxRangePushA(name); }
+  ~TraceRange() { nvtxRangePop(); }
+  TraceRange(const TraceRange&) = delete;
+  TraceRange& operator=(const TraceRange&) = delete;
+};
 
 // ---------------------------------------------------------------- host side
 

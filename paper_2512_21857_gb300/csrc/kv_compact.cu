@@ -154,6 +154,7 @@ adt_status adt_kv_compact(adt_bf16* k_cache, adt_bf16* v_cache, const int32_t* k
                           int32_t num_layers, int32_t max_kv, int64_t cache_layer_stride,
                           int64_t cache_stride_b, int64_t cache_stride_h,
                           int64_t tree_layer_stride, void* stream) {
+  adt::TraceRange trace_("adt_kv_compact");
   ADT_REQUIRE(k_cache && v_cache && kv_len && k_tree && v_tree && node_offsets && path && accept_len);
   ADT_REQUIRE(B >= 1 && B <= 65535 && Hkv >= 1 && num_layers >= 1 && num_layers <= 65535);
   ADT_REQUIRE(max_path >= 1 && max_path <= (1 << 20) && max_kv >= 1);
@@ -203,6 +204,7 @@ adt_status adt_kv_compact_inplace(adt_bf16* k_cache, adt_bf16* v_cache, const in
                                   int32_t max_path, const int32_t* accept_len, int32_t B, int32_t Hkv, int32_t D,
                                   int32_t num_layers, int32_t max_kv, int64_t cache_layer_stride,
                                   int64_t cache_stride_b, int64_t cache_stride_h, void* stream) {
+  adt::TraceRange trace_("adt_kv_compact_inplace");
   ADT_REQUIRE(k_cache && v_cache && kv_len && node_offsets && path && accept_len);
   ADT_REQUIRE(B >= 1 && B <= 65535 && Hkv >= 1 && Hkv <= 65535 && num_layers >= 1 && num_layers <= 65535);
   ADT_REQUIRE(max_path >= 1 && max_kv >= 1);

@@ -615,6 +615,7 @@ adt_status adt_tree_accept(const float* target_logits, int64_t ld_target,
                            float temperature, int32_t* path, int32_t max_path,
                            int32_t* accept_len, int32_t* bonus_token, void* workspace,
                            size_t workspace_bytes, void* stream) {
+  adt::TraceRange trace_("adt_tree_accept");
   return accept_impl(target_logits, nullptr, ld_target, draft_logits, nullptr, ld_draft, draft_row, 0.f, tokens,
                      parents, node_offsets, B, V, max_nodes, u_accept, u_sample, mode, temperature, path, max_path,
                      accept_len, bonus_token, workspace, workspace_bytes, stream);
@@ -628,6 +629,7 @@ adt_status adt_tree_accept_cfg(const float* target_cond, const float* target_unc
                                adt_accept_mode mode, float temperature, int32_t* path, int32_t max_path,
                                int32_t* accept_len, int32_t* bonus_token, void* workspace,
                                size_t workspace_bytes, void* stream) {
+  adt::TraceRange trace_("adt_tree_accept_cfg");
   ADT_REQUIRE(target_uncond);
   return accept_impl(target_cond, target_uncond, ld_target, draft_cond, draft_uncond, ld_draft, draft_row,
                      cfg_scale, tokens, parents, node_offsets, B, V, max_nodes, u_accept, u_sample, mode,

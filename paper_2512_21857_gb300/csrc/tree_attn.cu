@@ -1217,6 +1217,7 @@ adt_status adt_tree_attn(const adt_bf16* q, const adt_bf16* k_cache, const adt_b
                          const int32_t* node_offsets, int32_t B, int32_t H, int32_t Hkv, int32_t D,
                          int32_t max_nodes, int32_t max_kv, float softmax_scale, adt_bf16* out,
                          float* lse, void* workspace, size_t workspace_bytes, void* stream) {
+  adt::TraceRange trace_("adt_tree_attn");
   adt_status st = check_args(q, k_cache, v_cache, kv_len, cache_stride_b, cache_stride_h, k_tree, v_tree, parents,
                              node_offsets, B, H, Hkv, D, max_nodes, max_kv, softmax_scale, out);
   if (st != ADT_OK) return st;
@@ -1295,6 +1296,7 @@ extern "C" adt_status adt_tree_attn_noalloc(const adt_bf16* q, const adt_bf16* k
                                             int32_t B, int32_t H, int32_t Hkv, int32_t D,
                                             int32_t max_nodes, int32_t max_kv, float softmax_scale,
                                             adt_bf16* out, float* lse, void* stream) {
+  adt::TraceRange trace_("adt_tree_attn_noalloc");
   adt_status st = check_args(q, k_cache, v_cache, kv_len, cache_stride_b, cache_stride_h, k_tree, v_tree, parents,
                              node_offsets, B, H, Hkv, D, max_nodes, max_kv, softmax_scale, out);
   if (st != ADT_OK) return st;

@@ -760,6 +760,7 @@ adt_status adt_tree_expand(const float* logits, int64_t ld, const float* frontie
                            int32_t* child_parent, int32_t* keep_idx, float* next_score,
                            int32_t* next_id, void* workspace, size_t workspace_bytes,
                            void* stream) {
+  adt::TraceRange trace_("adt_tree_expand");
   return expand_impl(logits, nullptr, 0.f, ld, frontier_score, frontier_id, F, V, k_child, k_keep, temperature,
                      child_id_base, child_token, child_logp, child_score, child_parent, keep_idx, next_score,
                      next_id, workspace, workspace_bytes, stream);
@@ -772,6 +773,7 @@ adt_status adt_tree_expand_cfg(const float* logits_cond, const float* logits_unc
                                float* child_score, int32_t* child_parent, int32_t* keep_idx,
                                float* next_score, int32_t* next_id, void* workspace,
                                size_t workspace_bytes, void* stream) {
+  adt::TraceRange trace_("adt_tree_expand_cfg");
   ADT_REQUIRE(logits_uncond);
   return expand_impl(logits_cond, logits_uncond, cfg_scale, ld, frontier_score, frontier_id, F, V, k_child,
                      k_keep, temperature, child_id_base, child_token, child_logp, child_score, child_parent,
@@ -789,6 +791,7 @@ adt_status adt_tree_rerank(const int32_t* cand_token, const float* cand_score,
                            int32_t n_nodes, int32_t* tokens, int32_t* parents,
                            int32_t* cand_index, int32_t* depth, void* workspace,
                            size_t workspace_bytes, void* stream) {
+  adt::TraceRange trace_("adt_tree_rerank");
   ADT_REQUIRE(cand_token && cand_score && cand_parent && root_token && tokens && parents);
   ADT_REQUIRE(C >= 1 && C <= 65536 && n_nodes >= 1 && n_nodes <= C + 1 && n_nodes <= 4096);
   const size_t need = adt_tree_rerank_workspace_size(C);
