@@ -415,6 +415,15 @@ adt_status adt_ctrl_next(adt_ctrl* ctrl, int32_t pos, int32_t* depth, int32_t* w
  * 0 <= accept_len <= depth; positions pos .. pos+accept_len remember (d, k);
  * *next_pos (may be NULL) = pos + accept_len + 1. */
 adt_status adt_ctrl_update(adt_ctrl* ctrl, int32_t pos, int32_t accept_len, int32_t* next_pos);
+/* Checkpoint / resume: the controller's whole state (parameters, grids,
+ * the previous tree's acceptance rate) as bytes.  adt_ctrl_state_size gives
+ * the size (0 for NULL); adt_ctrl_save writes it into buf (bytes >= size);
+ * adt_ctrl_load creates a controller from saved bytes (freed by
+ * adt_ctrl_destroy), rejecting buffers that are short or not a saved
+ * state.  Host byte order: a checkpoint for the same build. */
+size_t adt_ctrl_state_size(const adt_ctrl* ctrl);
+adt_status adt_ctrl_save(const adt_ctrl* ctrl, void* buf, size_t bytes);
+adt_status adt_ctrl_load(const void* buf, size_t bytes, adt_ctrl** out);
 /* The (d, k) recorded for a generated position (0, 0 if not generated). */
 adt_status adt_ctrl_get(const adt_ctrl* ctrl, int32_t pos, int32_t* depth, int32_t* width);
 

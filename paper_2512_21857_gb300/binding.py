@@ -31,6 +31,7 @@ EXPORTED = [
     "adt_tree_accept_workspace_size", "adt_tree_accept", "adt_tree_accept_cfg",
     "adt_kv_compact", "adt_kv_compact_inplace",
     "adt_ctrl_create", "adt_ctrl_destroy", "adt_ctrl_next", "adt_ctrl_update", "adt_ctrl_get",
+    "adt_ctrl_state_size", "adt_ctrl_save", "adt_ctrl_load",
 ]
 
 
@@ -77,6 +78,9 @@ _SIGS = {
                                 _P], _I32),
     "adt_ctrl_create": ([ctypes.POINTER(CtrlParams), _I32, _I32, ctypes.POINTER(_P)], _I32),
     "adt_ctrl_destroy": ([_P], None),
+    "adt_ctrl_state_size": ([_P], _SZ),
+    "adt_ctrl_save": ([_P, _P, _SZ], _I32),
+    "adt_ctrl_load": ([_P, _SZ, ctypes.POINTER(_P)], _I32),
     "adt_ctrl_next": ([_P, _I32, ctypes.POINTER(_I32), ctypes.POINTER(_I32)], _I32),
     "adt_ctrl_update": ([_P, _I32, _I32, ctypes.POINTER(_I32)], _I32),
     "adt_ctrl_get": ([_P, _I32, ctypes.POINTER(_I32), ctypes.POINTER(_I32)], _I32),
@@ -307,6 +311,22 @@ class Controller:
         d, k = ctypes.c_int32(), ctypes.c_int32()
         _check(lib().adt_ctrl_get(self._h, pos, ctypes.byref(d), ctypes.byref(k)), "adt_ctrl_get")
         return d.value, k.value
+
+    def save(self) -> bytes:
+        """The controller's state as bytes (checkpoint)."""
+        n = int(lib().adt_ctrl_state_size(self._h))
+        buf = ctypes.create_string_buffer(n)
+        _check(lib().adt_ctrl_save(self._h, buf, n), "adt_ctrl_save")
+        return buf.raw
+
+    @classmethod
+    def load(cls, state: bytes) -> "Controller":
+        """A controller resumed from save()'s bytes."""
+        h = ctypes.c_void_p()
+        _check(lib().adt_ctrl_load(state, len(state), ctypes.byref(h)), "adt_ctrl_load")
+        obj = cls.__new__(cls)
+        obj._h = h
+        return obj
 
     def __del__(self):
         h = getattr(self, "_h", None)

@@ -2,6 +2,7 @@
 // initialisation, Eq. 2 bisectional adaptation, the bounds at the end of
 // Sec. 4.2, hyper-parameters of Sec. 5.1).  One object per image; no GPU.
 #include <cstdint>
+#include <cstring>
 #include <new>
 #include <vector>
 
@@ -161,6 +162,72 @@ adt_status adt_ctrl_update(adt_ctrl* c, int32_t pos, int32_t accept_len, int32_t
     c->k_grid[t] = c->cur_k;
   }
   if (next_pos) *next_pos = pos + accept_len + 1;
+  return ADT_OK;
+}
+
+// Saved state: a header, the parameters, the adaptation state and the two
+// grids, in host byte order (a checkpoint for the same build, not an
+// interchange format).
+namespace {
+constexpr uint32_t kStateMagic = 0x41445443u;  // "ADTC"
+constexpr uint32_t kStateVersion = 1u;
+struct StateHeader {
+  uint32_t magic, version;
+  int32_t h, w;
+  adt_ctrl_params p;
+  double alpha_prev;
+  int32_t have_alpha, have_cur, cur_d, cur_k;
+};
+}  // namespace
+
+size_t adt_ctrl_state_size(const adt_ctrl* c) {
+  if (!c) return 0;
+  return sizeof(StateHeader) + 2 * c->d_grid.size() * sizeof(int32_t);
+}
+
+adt_status adt_ctrl_save(const adt_ctrl* c, void* buf, size_t bytes) {
+  if (!c || !buf || bytes < adt_ctrl_state_size(c)) return ADT_ERR_INVALID_ARG;
+  StateHeader hd;
+  std::memset(&hd, 0, sizeof(hd));
+  hd.magic = kStateMagic;
+  hd.version = kStateVersion;
+  hd.h = c->h;
+  hd.w = c->w;
+  hd.p = c->p;
+  hd.alpha_prev = c->alpha_prev;
+  hd.have_alpha = c->have_alpha ? 1 : 0;
+  hd.have_cur = c->have_cur ? 1 : 0;
+  hd.cur_d = c->cur_d;
+  hd.cur_k = c->cur_k;
+  uint8_t* out = static_cast<uint8_t*>(buf);
+  std::memcpy(out, &hd, sizeof(hd));
+  const size_t g = c->d_grid.size() * sizeof(int32_t);
+  std::memcpy(out + sizeof(hd), c->d_grid.data(), g);
+  std::memcpy(out + sizeof(hd) + g, c->k_grid.data(), g);
+  return ADT_OK;
+}
+
+adt_status adt_ctrl_load(const void* buf, size_t bytes, adt_ctrl** out) {
+  if (!buf || !out || bytes < sizeof(StateHeader)) return ADT_ERR_INVALID_ARG;
+  StateHeader hd;
+  std::memcpy(&hd, buf, sizeof(hd));
+  if (hd.magic != kStateMagic || hd.version != kStateVersion || hd.h < 1 || hd.w < 1 ||
+      static_cast<int64_t>(hd.h) * hd.w > (int64_t{1} << 28))
+    return ADT_ERR_INVALID_ARG;
+  const size_t g = static_cast<size_t>(hd.h) * hd.w * sizeof(int32_t);
+  if (bytes < sizeof(hd) + 2 * g) return ADT_ERR_INVALID_ARG;
+  adt_ctrl* c = nullptr;
+  adt_status st = adt_ctrl_create(&hd.p, hd.h, hd.w, &c);  // validates the parameters
+  if (st != ADT_OK) return st;
+  const uint8_t* in = static_cast<const uint8_t*>(buf);
+  std::memcpy(c->d_grid.data(), in + sizeof(hd), g);
+  std::memcpy(c->k_grid.data(), in + sizeof(hd) + g, g);
+  c->alpha_prev = hd.alpha_prev;
+  c->have_alpha = hd.have_alpha != 0;
+  c->have_cur = hd.have_cur != 0;
+  c->cur_d = hd.cur_d;
+  c->cur_k = hd.cur_k;
+  *out = c;
   return ADT_OK;
 }
 

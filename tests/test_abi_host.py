@@ -152,3 +152,33 @@ def test_guidance_entry_points_check_their_extra_arguments(lib):
                                    8, f, f, None, 0, None) == 1
     assert lib.adt_tree_accept_cfg(f, f, 128, f, None, 128, None, 3.0, f, f, f, 1, 100, 8, f, f, 1, 1.0, f, 8, f, f,
                                    None, 0, None) == 1
+
+
+def test_controller_checkpoint_resume(lib):
+    """A controller saved mid-image and loaded again makes the same choices
+    as the one that kept running."""
+    params = dict(beta=1.0, l_d=1, l_k=3, d_lo=1, d_hi=9, k_lo=4, k_hi=13, init_mode=B.INIT_TOKENFLOCK, seed=5)
+    g = np.random.default_rng(9)
+    accepts = g.integers(0, 10, size=200).tolist()
+    a = B.Controller(24, 24, **params)
+    pos = 0
+    for x in accepts[:60]:
+        d, _ = a.next(pos)
+        pos = a.update(pos, min(x, d))
+    state = a.save()
+    b = B.Controller.load(state)
+    pos_a = pos_b = pos
+    for x in accepts[60:]:
+        if pos_a >= 24 * 24:
+            break
+        da = a.next(pos_a)
+        assert b.next(pos_b) == da
+        pos_a = a.update(pos_a, min(x, da[0]))
+        pos_b = b.update(pos_b, min(x, da[0]))
+    for p in range(24 * 24):
+        assert a.get(p) == b.get(p)
+    # short or foreign buffers are rejected
+    with pytest.raises(B.AdtError):
+        B.Controller.load(state[:40])
+    with pytest.raises(B.AdtError):
+        B.Controller.load(b"\0" * len(state))
