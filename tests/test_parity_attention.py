@@ -84,6 +84,18 @@ def test_7b_shape_one_layer_full_size():
     assert np.abs(lse - ref_lse).max() < LSE_ATOL
 
 
+@pytest.mark.parametrize("sizes,kv,H,D", [
+    ([64], [16384], 8, 128),        # 19 splits of 7 chunks each, merged through the workspace
+    ([64, 40], [8192, 7000], 32, 128),  # 2 splits per head: 33-chunk pipelines, many barrier phases
+])
+def test_long_prefixes(sizes, kv, H, D):
+    case = AttnCase(sizes, kv, H, H, D, seed=17 + len(sizes), lmax=max(kv) + 8)
+    got, lse, _ = case.run_gpu(max_nodes=64, max_kv=max(kv) + 8)
+    ref, ref_lse = case.run_oracle()
+    assert_attention_close(got, ref)
+    assert np.abs(lse - ref_lse).max() < LSE_ATOL
+
+
 def test_batch_of_eight_ragged_prefixes():
     g = np.random.default_rng(5)
     kv = g.integers(600, 2401, size=8).tolist()
