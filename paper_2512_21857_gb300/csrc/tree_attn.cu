@@ -307,58 +307,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int qt = kLarge ? static_cast<int>(blockIdx.z) % p.qtiles : 0;
   const int g = h / p.group;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-
-  // Programmatic dependent launch: every global-memory access comes after
-  // the previous kernel in the stream has completed (immediate when this
-  // launch does not overlap one).
-  asm volatile("griddepcontrol.wait;\n" ::: "memory");
-  const int node0 = p.offs[b];
-  const int n = p.offs[b + 1] - node0;
-  const int total_nodes = p.offs[p.B];
-  const int L = p.kv_len[b];
-
-  // Conditions that hold for every CTA of this (tree, head, tile): all
-  // leave here.  A tile past the end of its tree has no rows.
-  if (n < 1 || n > kMaxNodes * (kLarge ? p.qtiles : 1) || node0 < 0 || node0 + n > total_nodes) {
-    if (split == 0 && h == 0 && qt == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_BAD_TREE);
-    return;
-  }
-  if (L < 0 || L > p.max_kv) {
-    if (split == 0 && h == 0 && qt == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_KV_RANGE);
-    return;
-  }
-  const int row0 = qt * kMaxNodes;  // first node (query row) of this tile
-  const int nq = min(n - row0, kMaxNodes);
-  if (nq <= 0) return;
-
-  // The keys are cut into chunks of two 64-key units: ceil(P / 2) prefix
-  // chunks (P = ceil(L / 64); the last holds one unit when P is odd), then
-  // the tree units the tile's rows can see, 0 .. qt (a node's ancestors come
-  // before it), two to a chunk.  Split s takes chunks [s T / S, (s + 1) T / S)
-  // of the T and processes its tree chunks first.
-  const int P = (L + kUnit - 1) / kUnit;
-  const int Pc = (P + 1) / 2;
-  const int Tc = kLarge ? (qt + 2) / 2 : 1;  // tree chunks of this tile
-  const int T = Pc + Tc;
-  const int S = p.splits;
-  const int c_begin = static_cast<int>(static_cast<int64_t>(split) * T / S);
-  const int c_end = static_cast<int>(static_cast<int64_t>(split + 1) * T / S);
-  const int nch = c_end - c_begin;
-  const int tc0 = max(c_begin, Pc) - Pc;         // first tree chunk of this split
-  const int n_tc = max(0, c_end - max(c_begin, Pc));  // its tree chunks, in slots 0 .. n_tc-1
   const int NS = C::kStages;
-  auto chunk_keys = [&](int j) -> int {
-    if (j < n_tc) return (kLarge && 2 * (tc0 + j) + 1 <= qt ? 2 : 1) * kUnit;
-    const int pc = c_begin + j - n_tc;
-    return (2 * pc + 1 < P ? 2 : 1) * kUnit;
-  };
-  auto chunk_key0 = [&](int j) -> int { return (c_begin + j - n_tc) * kChunk; };
 
-  uint8_t* sQ = smem + C::kQOff;
-  uint8_t* sP = smem + C::kPOff;
-  uint8_t* sStage = smem + C::kStageOff;
-  float* slots = reinterpret_cast<float*>(smem + C::kSlotOff);  // merge: [S][rows_per][kRowStride]
-
+  // Set-up that touches no memory the previous kernel writes: the
+  // mbarriers, the tensor memory and the tensor maps' descriptors.  It runs
+  // before the dependency wait, so a CTA that is resident early (on an SM
+  // the previous launch leaves idle) has it done when the wait releases.
   if (tid == 0) {
     s_bad = 0;
     s_abort = 0;
@@ -383,6 +337,63 @@ __global__ void __launch_bounds__(kThreads, 1)
     sm100::tmem_alloc(sm100::smem_addr(&tmem_slot), kTmemCols);
     sm100::tmem_relinquish();
   }
+  if ((warp == kKLoadWarp || warp == kVLoadWarp) && lane == 0)
+    sm100::prefetch_tensormap(warp == kVLoadWarp ? &tm_v : &tm_k);
+  sm100::tc_fence_before();
+  __syncthreads();
+  sm100::tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+
+  // Programmatic dependent launch: every global-memory access comes after
+  // the previous kernel in the stream has completed (immediate when this
+  // launch does not overlap one).
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
+  const int node0 = p.offs[b];
+  const int n = p.offs[b + 1] - node0;
+  const int total_nodes = p.offs[p.B];
+  const int L = p.kv_len[b];
+
+  // Conditions that hold for every CTA of this (tree, head, tile): all
+  // leave here, handing back the tensor memory.  A tile past the end of its
+  // tree has no rows.
+  const int row0 = qt * kMaxNodes;  // first node (query row) of this tile
+  const bool bad_tree = n < 1 || n > kMaxNodes * (kLarge ? p.qtiles : 1) || node0 < 0 || node0 + n > total_nodes;
+  const bool bad_kv = L < 0 || L > p.max_kv;
+  if (bad_tree || bad_kv || n - row0 <= 0) {
+    if (split == 0 && h == 0 && qt == 0 && tid == 0 && (bad_tree || bad_kv))
+      adt::raise_error(p.err, bad_tree ? ADT_DEVERR_BAD_TREE : ADT_DEVERR_KV_RANGE);
+    if (warp == 0) sm100::tmem_dealloc(tmem, kTmemCols);
+    return;
+  }
+  const int nq = min(n - row0, kMaxNodes);
+
+  // The keys are cut into chunks of two 64-key units: ceil(P / 2) prefix
+  // chunks (P = ceil(L / 64); the last holds one unit when P is odd), then
+  // the tree units the tile's rows can see, 0 .. qt (a node's ancestors come
+  // before it), two to a chunk.  Split s takes chunks [s T / S, (s + 1) T / S)
+  // of the T and processes its tree chunks first.
+  const int P = (L + kUnit - 1) / kUnit;
+  const int Pc = (P + 1) / 2;
+  const int Tc = kLarge ? (qt + 2) / 2 : 1;  // tree chunks of this tile
+  const int T = Pc + Tc;
+  const int S = p.splits;
+  const int c_begin = static_cast<int>(static_cast<int64_t>(split) * T / S);
+  const int c_end = static_cast<int>(static_cast<int64_t>(split + 1) * T / S);
+  const int nch = c_end - c_begin;
+  const int tc0 = max(c_begin, Pc) - Pc;         // first tree chunk of this split
+  const int n_tc = max(0, c_end - max(c_begin, Pc));  // its tree chunks, in slots 0 .. n_tc-1
+  auto chunk_keys = [&](int j) -> int {
+    if (j < n_tc) return (kLarge && 2 * (tc0 + j) + 1 <= qt ? 2 : 1) * kUnit;
+    const int pc = c_begin + j - n_tc;
+    return (2 * pc + 1 < P ? 2 : 1) * kUnit;
+  };
+  auto chunk_key0 = [&](int j) -> int { return (c_begin + j - n_tc) * kChunk; };
+
+  uint8_t* sQ = smem + C::kQOff;
+  uint8_t* sP = smem + C::kPOff;
+  uint8_t* sStage = smem + C::kStageOff;
+  float* slots = reinterpret_cast<float*>(smem + C::kSlotOff);  // merge: [S][rows_per][kRowStride]
+
   if (warp < kSoftmaxWarps) {
     // Q tile: rows row0 .. row0+63 of the tree (rows past it zero-filled);
     // this split's tree chunks (K/V of kv head g, nodes past the tree
@@ -415,10 +426,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     static_assert(C::kOnesBytes == kSoftmaxWarps * 32 * 16, "one 16-byte store per softmax thread");
     reinterpret_cast<uint4*>(smem + C::kOnesOff)[tid] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
   }
-  sm100::tc_fence_before();
+  // Q's copies are requested before the stage loads: a CTA's first stages
+  // are 128 KB, and Q queued behind them would hold back the first S.
   __syncthreads();
-  sm100::tc_fence_after();
-  const uint32_t tmem = tmem_slot;
   // The mbarriers are initialised: tell the cluster (the merge's bulk copies
   // complete on a peer's barrier; every thread waits on this before one).
   sm100::cluster_arrive_relaxed();
