@@ -29,36 +29,49 @@ struct CompactParams {
   unsigned* err;
 };
 
+// Warp 0: checks path entries 0 .. a of one tree at once (lane j reads
+// entries j, j + 32, ...): each a node of the tree (0 <= node < n), the first
+// the root.  Entry `want` goes to *want_node, and with keep_all every entry
+// to keep[j].  Returns the same verdict in every lane.
+__device__ __forceinline__ bool warp_check_path(const int32_t* path, int a, int n, int want, int* want_node,
+                                                int* keep) {
+  const int lane = threadIdx.x & 31;
+  bool bad = false;
+  for (int j = lane; j <= a; j += 32) {
+    const int node = path[j];
+    bad |= node < 0 || node >= n || (j == 0 && node != 0);
+    if (j == want) *want_node = node;
+    if (keep) keep[j] = node;
+  }
+  return !__any_sync(adt::kFullMask, bad);
+}
+
 __global__ void __launch_bounds__(kThreads) kv_compact_kernel(const CompactParams p) {
-  __shared__ int s_ok;
+  __shared__ int s_ok, s_node;
   adt::pdl_wait_then_release();
   const int i = blockIdx.x, b = blockIdx.y, l = blockIdx.z, tid = threadIdx.x;
   const int a = p.alen[b];
   const int L = p.kv_len[b];
   const int node0 = p.offs[b];
   const int n = p.offs[b + 1] - node0;
-  if (tid == 0) {
+  if (tid < 32) {
     int ok = (a >= 0 && a < p.max_path && L >= 0 && static_cast<int64_t>(L) + a + 1 <= p.max_kv) ? 1 : 0;
     unsigned bits = ok ? 0u : ADT_DEVERR_KV_RANGE;
-    if (ok) {
-      for (int j = 0; j <= a; ++j) {
-        const int node = p.path[static_cast<int64_t>(b) * p.max_path + j];
-        if (node < 0 || node >= n || (j == 0 && node != 0)) {
-          ok = 0;
-          bits = ADT_DEVERR_BAD_PATH;
-          break;
-        }
-      }
+    if (ok && !warp_check_path(p.path + static_cast<int64_t>(b) * p.max_path, a, n, i, &s_node, nullptr)) {
+      ok = 0;
+      bits = ADT_DEVERR_BAD_PATH;
     }
-    s_ok = ok;
-    if (i == 0 && l == 0) {
-      if (!ok) adt::raise_error(p.err, bits);
-      if (p.kv_len_out) p.kv_len_out[b] = ok ? L + a + 1 : L;
+    if (tid == 0) {
+      s_ok = ok;
+      if (i == 0 && l == 0) {
+        if (!ok) adt::raise_error(p.err, bits);
+        if (p.kv_len_out) p.kv_len_out[b] = ok ? L + a + 1 : L;
+      }
     }
   }
   __syncthreads();
   if (!s_ok || i > a) return;
-  const int node = node0 + p.path[static_cast<int64_t>(b) * p.max_path + i];
+  const int node = node0 + s_node;
   const int vec_per_head = p.D / 8;  // 16-byte vectors of bf16
   const int nvec = p.Hkv * vec_per_head;
   const int64_t src = (static_cast<int64_t>(l) * p.tls + static_cast<int64_t>(node) * p.Hkv * p.D) / 8;
@@ -93,32 +106,28 @@ struct InplaceParams {
 
 __global__ void __launch_bounds__(kThreads) kv_compact_inplace_kernel(const InplaceParams p) {
   extern __shared__ uint4 stage[];  // [row i][K, V][D / 8]
-  __shared__ int s_ok;
+  __shared__ int s_ok, s_unused;
+  __shared__ int path[kMaxInplacePath];  // the tree's path entries 0 .. a
   adt::pdl_wait_then_release();
   const int g = blockIdx.x, b = blockIdx.y, l = blockIdx.z, tid = threadIdx.x;
   const int a = p.alen[b];
   const int L = p.kv_len[b];
   const int n = p.offs[b + 1] - p.offs[b];
-  const int32_t* path = p.path + static_cast<int64_t>(b) * p.max_path;
-  if (tid == 0) {
+  if (tid < 32) {
     // the tree's rows L .. L+n-1 and the path's destinations must fit
     int ok = (a >= 0 && a < p.max_path && L >= 0 && n >= 1 && a < n &&
               static_cast<int64_t>(L) + n <= p.max_kv) ? 1 : 0;
     unsigned bits = ok ? 0u : ADT_DEVERR_KV_RANGE;
-    if (ok) {
-      for (int j = 0; j <= a; ++j) {
-        const int node = path[j];
-        if (node < 0 || node >= n || (j == 0 && node != 0)) {
-          ok = 0;
-          bits = ADT_DEVERR_BAD_PATH;
-          break;
-        }
-      }
+    if (ok && !warp_check_path(p.path + static_cast<int64_t>(b) * p.max_path, a, n, -1, &s_unused, path)) {
+      ok = 0;
+      bits = ADT_DEVERR_BAD_PATH;
     }
-    s_ok = ok;
-    if (g == 0 && l == 0) {
-      if (!ok) adt::raise_error(p.err, bits);
-      if (p.kv_len_out) p.kv_len_out[b] = ok ? L + a + 1 : L;
+    if (tid == 0) {
+      s_ok = ok;
+      if (g == 0 && l == 0) {
+        if (!ok) adt::raise_error(p.err, bits);
+        if (p.kv_len_out) p.kv_len_out[b] = ok ? L + a + 1 : L;
+      }
     }
   }
   __syncthreads();

@@ -232,7 +232,6 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
   __shared__ __align__(8) uint64_t s_bar;
   __shared__ int s_last;
   __shared__ double s_lse;
-  adt::pdl_wait_then_release();
   uint64_t* cross_s = cand;  // cross-row keys (reuses the candidate buffer)
   uint64_t* sel = cand;      // radix path [kMaxKeep]
 
@@ -240,6 +239,16 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
   const int rank = blockIdx.x, C = gridDim.x, r = blockIdx.y;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int K = p.k;
+  // Shared-memory set-up before the dependency wait (it reads nothing an
+  // earlier kernel writes): after the wait the first bulk copy goes out at once.
+  for (int i = tid; i < kMaxK; i += kThreads) ctl[i] = 0ull;
+  if (tid == 0) {
+    s_cnt = 0u;
+    sm100::mbar_init(sm100::smem_addr(&s_bar), 1);
+    sm100::fence_mbar_init();
+  }
+  __syncthreads();
+  adt::pdl_wait_then_release();
   // This CTA's share of the row: [c0, c1), c0 a multiple of 4.
   const int per = (((p.V + C - 1) / C) + 3) & ~3;
   const int c0 = min(p.V, rank * per), c1 = min(p.V, c0 + per);
@@ -253,13 +262,6 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
   const bool writer = rank == 0 && tid < K;
   const float f_score = writer ? p.fscore[r] : 0.f;
   const int32_t f_id = writer ? (p.fid ? p.fid[r] : r) : 0;
-  for (int i = tid; i < kMaxK; i += kThreads) ctl[i] = 0ull;
-  if (tid == 0) {
-    s_cnt = 0u;
-    sm100::mbar_init(sm100::smem_addr(&s_bar), 1);
-    sm100::fence_mbar_init();
-  }
-  __syncthreads();
   uint32_t phase = 0;
   bool ok = true;
 
