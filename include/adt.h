@@ -264,7 +264,11 @@ adt_status adt_tree_rerank(const int32_t* cand_token, const float* cand_score,
  * target_logits [device] fp32, row of global node n at target + n*ld_target.
  * draft_logits  [device] fp32 (SPEC only, else may be NULL); the draft row
  *         of node n is draft + draft_row[n]*ld_draft, or + n*ld_draft when
- *         draft_row is NULL.
+ *         draft_row is NULL.  Only nodes with children have their draft row
+ *         read: a leaf may map to -1.  A node with children and a negative
+ *         draft_row sets ADT_DEVERR_BAD_INDEX and the walk stops there, its
+ *         bonus drawn from the target distribution; non-negative rows are
+ *         not range-checked (each must be a row of draft_logits).
  * tokens, parents [device] int32 [Ntot]; node_offsets [device] int32 [B+1].
  * u_accept, u_sample [device] fp32 [Ntot] in [0, 1) (SPEC modes; GREEDY may
  *         pass NULL): u_accept[n] decides child n, u_sample[v] draws the

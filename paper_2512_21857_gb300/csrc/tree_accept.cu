@@ -310,7 +310,7 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
       }
       __syncthreads();
     }
-    const int nk = sh.nkids;
+    int nk = sh.nkids;
     const int gv = node0 + v;
     const float* trow = p.target + static_cast<int64_t>(gv) * p.ldt;
     const float* trow_u = p.target_u ? p.target_u + static_cast<int64_t>(gv) * p.ldt : nullptr;
@@ -361,12 +361,18 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
 
     // ---- sampling modes: p = softmax(target row / T) in the slices.
     const bool spec = p.mode == ADT_ACCEPT_SPEC;
+    // The draft row of v (the same value in every thread of the cluster).  A
+    // node with children but no draft row (negative index) is an error; its
+    // children are then not considered and the bonus comes from p.
+    const int64_t dr = spec && nk > 0 && p.drow ? static_cast<int64_t>(p.drow[gv]) : gv;
+    if (dr < 0) {
+      if (w.rank == 0 && tid == 0) adt::raise_error(p.err, ADT_DEVERR_BAD_INDEX);
+      nk = 0;
+    }
     const bool need_q = spec && nk > 0;
     load_slice(trow, trow_u, lo, cnt, p.Vs, pbuf, p);
-    if (need_q) {
-      const int64_t dr = p.drow ? p.drow[gv] : gv;
+    if (need_q)
       load_slice(p.draft + dr * p.ldd, p.draft_u ? p.draft_u + dr * p.ldd : nullptr, lo, cnt, p.Vs, qbuf, p);
-    }
     __syncthreads();
     const float mp = slice_max(pbuf, p.Vs, &sh);
     const float mq = need_q ? slice_max(qbuf, p.Vs, &sh) : 0.f;

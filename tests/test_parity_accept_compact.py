@@ -109,6 +109,34 @@ def test_spec_uses_draft_row_mapping():
     compare(tb, res, path, alen, bonus)
 
 
+def test_spec_leaves_may_have_no_draft_row_and_a_missing_row_is_flagged():
+    """Leaves map to draft row -1 (their rows are never read): the walk is the
+    oracle's.  The root without a draft row is flagged, accepts nothing and
+    draws its bonus from its own target distribution, as a lone root would."""
+    V, n = 16384, 20
+    tb = synth.tree_batch([n], V, 8)
+    target, draft = make_rows(tb, V, 8, 0.3)
+    ua, us = synth.uniforms(n, 8, "ua"), synth.uniforms(n, 8, "us")
+    has_kids = np.zeros(n, dtype=bool)
+    has_kids[tb.parents[1:]] = True
+    mapping = np.where(has_kids, np.arange(n), -1).astype(np.int32)
+    res = oracle.tree_accept(target, draft, tb.tokens, tb.parents, tb.node_offsets, B.ACCEPT_SPEC, ua, us)
+    assert res["min_margin"] > ACCEPT_MARGIN
+    B.adt_get_device_error()
+    path, alen, bonus = run_accept_gpu(target, draft, tb, B.ACCEPT_SPEC, ua, us, draft_row=mapping)
+    compare(tb, res, path, alen, bonus)
+    assert B.adt_get_device_error() == 0
+
+    mapping[0] = -1
+    lone = oracle.tree_accept(target[:1], draft[:1], tb.tokens[:1], tb.parents[:1], np.array([0, 1]),
+                              B.ACCEPT_SPEC, ua[:1], us[:1])
+    assert lone["sample_margin"] > SAMPLE_MARGIN
+    path, alen, bonus = run_accept_gpu(target, draft, tb, B.ACCEPT_SPEC, ua, us, draft_row=mapping)
+    assert B.adt_get_device_error() & B.DEVERR_BAD_INDEX
+    assert alen[0] == 0 and path[0, 0] == 0 and (path[0, 1:] == -1).all()
+    assert bonus[0] == lone["bonus"][0]
+
+
 def test_path_longer_than_buffer_is_cut_and_flagged():
     V = 1000
     tb = synth.tree_batch([12], V, 3, chain=True)
