@@ -303,7 +303,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ volatile int s_abort;
 
   const int split = blockIdx.x, h = blockIdx.y;
-  const int b = kLarge ? static_cast<int>(blockIdx.z) / p.qtiles : static_cast<int>(blockIdx.z);
+  const int slot = kLarge ? static_cast<int>(blockIdx.z) / p.qtiles : static_cast<int>(blockIdx.z);
   const int qt = kLarge ? static_cast<int>(blockIdx.z) % p.qtiles : 0;
   const int g = h / p.group;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -348,10 +348,36 @@ __global__ void __launch_bounds__(kThreads, 1)
   // the previous kernel in the stream has completed (immediate when this
   // launch does not overlap one).
   asm volatile("griddepcontrol.wait;\n" ::: "memory");
-  const int node0 = p.offs[b];
-  const int n = p.offs[b + 1] - node0;
-  const int total_nodes = p.offs[p.B];
-  const int L = p.kv_len[b];
+  // The tree of this CTA.  With several trees (up to 32) the launch slots
+  // go to the trees by decreasing prefix length (ties: lower index): the
+  // CTAs are dispatched in slot order, so the longest streams start first
+  // and the short ones fill in behind them instead of a late long tree
+  // ending the launch.  Every warp ranks the trees itself (one lane per
+  // tree), from the same single round of loads the one-tree path makes.
+  int b, node0, n, total_nodes, L;
+  if (p.B > 1 && p.B <= 32) {
+    const bool mine = lane < p.B;
+    const int kl = mine ? p.kv_len[lane] : 0;
+    const int off = mine ? p.offs[lane] : 0;
+    total_nodes = p.offs[p.B];
+    int rank = 0;
+    for (int i = 0; i < p.B; ++i) {
+      const int o = __shfl_sync(adt::kFullMask, kl, i);
+      rank += (o > kl || (o == kl && i < lane)) ? 1 : 0;
+    }
+    const unsigned hit = __ballot_sync(adt::kFullMask, mine && rank == slot);
+    b = hit ? __ffs(hit) - 1 : slot;
+    L = __shfl_sync(adt::kFullMask, kl, b);
+    node0 = __shfl_sync(adt::kFullMask, off, b);
+    const int next = __shfl_sync(adt::kFullMask, off, (b + 1) & 31);
+    n = (b + 1 < p.B ? next : total_nodes) - node0;
+  } else {
+    b = slot;
+    node0 = p.offs[b];
+    n = p.offs[b + 1] - node0;
+    total_nodes = p.offs[p.B];
+    L = p.kv_len[b];
+  }
 
   // Conditions that hold for every CTA of this (tree, head, tile): all
   // leave here, handing back the tensor memory.  A tile past the end of its
