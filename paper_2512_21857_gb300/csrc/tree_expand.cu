@@ -514,14 +514,34 @@ struct RerankParams {
 // candidate is selected when fewer than n_nodes - 1 candidate keys exceed
 // its own (a warp takes a key and its lanes count), node ids follow
 // ascending candidate index (block scan of the selection flags), and the
-// node maps, parents and depths never leave shared memory.
+// node maps, parents and depths never leave shared memory.  With at most
+// kRerankBound nodes to select from at least 64 candidates, only the keys
+// at or above a bound are ranked: every warp's two largest keys (over a
+// strided view, so that every warp holds candidates) give 64 distinct keys,
+// and the (n_nodes - 1)-th largest of them has at least n_nodes - 1 keys at
+// or above it.
 constexpr int kRerankSmall = 1024;
+constexpr int kRerankBound = 64;
+
+__device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const uint64_t w = __shfl_xor_sync(adt::kFullMask, v, o);
+    v = w > v ? w : v;
+  }
+  return v;
+}
 
 __global__ void __launch_bounds__(kRerankThreads) rerank_small_kernel(const RerankParams p) {
   __shared__ uint64_t keys[kRerankSmall];
   __shared__ int node_of[kRerankSmall];
   __shared__ int cand_of_node[kRerankSmall + 1];
   __shared__ int par[kRerankSmall + 1];
+  __shared__ int cpar_s[kRerankSmall];
+  __shared__ uint64_t list[kRerankSmall];
+  __shared__ uint64_t s_top[2 * 32];
+  __shared__ uint64_t s_bound;
+  __shared__ int s_nlist;
   __shared__ int warp_tot[32];
   __shared__ int s_bad;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -534,20 +554,62 @@ __global__ void __launch_bounds__(kRerankThreads) rerank_small_kernel(const Rera
     if (p.depth) p.depth[0] = 0;
     par[0] = -1;
     s_bad = 0;
+    s_nlist = 0;
   }
   if (need == 0) return;
-  for (int i = tid; i < C; i += kRerankThreads) keys[i] = adt::select_key(p.cscore[i], static_cast<uint32_t>(i));
-  __syncthreads();
-  // selection flag of candidate i (one per thread: C <= kRerankThreads)
-  bool sel = false;
-  for (int i = warp; i < C; i += kRerankThreads / 32) {
-    const uint64_t key = keys[i];
-    int rk = 0;
-    for (int j = 0; j < C; j += 32) rk += __popc(__ballot_sync(adt::kFullMask, j + lane < C && keys[j + lane] > key));
-    if (lane == 0) node_of[i] = rk < need ? 1 : 0;
+  // Candidate tid (C <= kRerankThreads): its key, token and parent id, all
+  // loaded in one round; node_of holds the selection flags until the scan.
+  uint64_t key = 0ull;
+  int tok = 0;
+  if (tid < C) {
+    key = adt::select_key(p.cscore[tid], static_cast<uint32_t>(tid));
+    tok = p.ctok[tid];
+    cpar_s[tid] = p.cpar[tid];
+    keys[tid] = key;
+    node_of[tid] = 0;
   }
   __syncthreads();
-  if (tid < C) sel = node_of[tid] != 0;
+  if (need <= kRerankBound && C >= 2 * 32) {
+    {
+      const int i = lane * 32 + warp;  // every warp sees at least two candidates
+      const uint64_t v = i < C ? keys[i] : 0ull;
+      const uint64_t m1 = warp_max_u64(v);
+      const uint64_t m2 = warp_max_u64(v == m1 ? 0ull : v);
+      if (lane == 0) {
+        s_top[warp] = m1;
+        s_top[warp + 32] = m2;
+      }
+    }
+    __syncthreads();
+    {
+      // warp w ranks s_top[w] and s_top[w + 32] among the 64
+      const uint64_t x = s_top[lane], y = s_top[lane + 32];
+      const uint64_t a = s_top[warp], c = s_top[warp + 32];
+      const int ra = __popc(__ballot_sync(adt::kFullMask, x > a)) + __popc(__ballot_sync(adt::kFullMask, y > a));
+      const int rc = __popc(__ballot_sync(adt::kFullMask, x > c)) + __popc(__ballot_sync(adt::kFullMask, y > c));
+      if (lane == 0 && ra == need - 1) s_bound = a;
+      if (lane == 0 && rc == need - 1) s_bound = c;
+    }
+    __syncthreads();
+    if (tid < C && key >= s_bound) list[atomicAdd(&s_nlist, 1)] = key;
+    __syncthreads();
+    const int nl = s_nlist;
+    for (int e = warp; e < nl; e += kRerankThreads / 32) {
+      const uint64_t ke = list[e];
+      int rk = 0;
+      for (int j = 0; j < nl; j += 32) rk += __popc(__ballot_sync(adt::kFullMask, j + lane < nl && list[j + lane] > ke));
+      if (lane == 0 && rk < need) node_of[adt::select_key_index(ke)] = 1;
+    }
+  } else {
+    for (int i = warp; i < C; i += kRerankThreads / 32) {
+      const uint64_t ki = keys[i];
+      int rk = 0;
+      for (int j = 0; j < C; j += 32) rk += __popc(__ballot_sync(adt::kFullMask, j + lane < C && keys[j + lane] > ki));
+      if (lane == 0) node_of[i] = rk < need ? 1 : 0;
+    }
+  }
+  __syncthreads();
+  const bool sel = tid < C && node_of[tid] != 0;
   // node id = 1 + selected candidates of lower index (block exclusive scan)
   const unsigned bal = __ballot_sync(adt::kFullMask, sel);
   if (lane == 0) warp_tot[warp] = __popc(bal);
@@ -559,13 +621,13 @@ __global__ void __launch_bounds__(kRerankThreads) rerank_small_kernel(const Rera
     node_of[tid] = node;
     if (sel) {
       cand_of_node[node] = tid;
-      p.tokens[node] = p.ctok[tid];
+      p.tokens[node] = tok;
       if (p.cand_index) p.cand_index[node] = tid;
     }
   }
   __syncthreads();
   for (int node = 1 + tid; node <= need; node += kRerankThreads) {
-    const int pc = p.cpar[cand_of_node[node]];
+    const int pc = cpar_s[cand_of_node[node]];
     int pr = 0;
     if (pc >= 0) {
       pr = pc < C ? node_of[pc] : -1;

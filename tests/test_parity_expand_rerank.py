@@ -181,9 +181,16 @@ def _random_pool(C, seed):
     return tok, sc, par
 
 
-@pytest.mark.parametrize("C,n", [(328, 64), (1534, 64), (5000, 4096), (9, 10), (70, 1)])
-def test_rerank_matches_oracle(C, n):
+@pytest.mark.parametrize("C,n", [(328, 64), (1534, 64), (5000, 4096), (9, 10), (70, 1),
+                                 (64, 65), (100, 65), (1024, 64), (600, 200), (63, 64), (1024, 1025)])
+@pytest.mark.parametrize("flat", [False, True])
+def test_rerank_matches_oracle(C, n, flat):
+    """Small pools select by a bound when n - 1 <= 64 and C >= 64, by full
+    ranking otherwise; pools past 1024 candidates take the radix kernel.
+    flat: every score equal, so the candidate index alone decides."""
     tok, sc, par = _random_pool(C, seed=C + n)
+    if flat:
+        sc = np.zeros_like(sc)
     dev = "cuda"
     res = dict(tokens=torch.empty(n, dtype=torch.int32, device=dev),
                parents=torch.empty(n, dtype=torch.int32, device=dev),
