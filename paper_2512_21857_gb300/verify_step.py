@@ -11,8 +11,12 @@ A step, for each image b of a batch (Sec. 3.1, Fig. 5, Eq. 4):
   5. adt_kv_compact commits the accepted path's K/V for all layers.
 Tree shapes (d_b, k_b) are host decisions (the controller, Sec. 4), so all
 launch shapes are known on the host and the whole step can be captured in a
-CUDA graph.  This module only allocates device memory (torch) and issues the
-library calls; every computation runs in the library's kernels.
+CUDA graph.  The images' draft phases (1-2) are independent chains of small,
+latency-bound launches: with more than one image each chain runs on its own
+stream, forked from the step's stream and joined back to it (in a captured
+graph, parallel branches).  This module only allocates device memory
+(torch) and issues the library calls; every computation runs in the
+library's kernels.
 """
 from __future__ import annotations
 
@@ -95,11 +99,13 @@ class TreeVerifyStep:
         self.pool_score = [torch.zeros(s.candidates(b), **f32) for b in range(Bn)]
         self.pool_logp = [torch.zeros(s.candidates(b), **f32) for b in range(Bn)]
         self.pool_par = [torch.zeros(s.candidates(b), **i32) for b in range(Bn)]
-        self.front_score = torch.zeros((2, kmax), **f32)
-        self.front_id = torch.full((2, kmax), -1, **i32)
+        # per image: the two alternating frontiers and the kept indices, so
+        # that the images' draft chains can run concurrently
+        self.front_score = [torch.zeros((2, kmax), **f32) for _ in range(Bn)]
+        self.front_id = [torch.full((2, kmax), -1, **i32) for _ in range(Bn)]
         self.root_score = torch.zeros(1, **f32)
         self.root_id = torch.full((1,), -1, **i32)
-        self.keep_idx = torch.zeros(kmax, **i32)
+        self.keep_idx = [torch.zeros(kmax, **i32) for _ in range(Bn)]
         self.tokens = torch.zeros(self.ntot, **i32)
         self.parents = torch.zeros(self.ntot, **i32)
         self.cand_index = torch.zeros(self.ntot, **i32)
@@ -111,10 +117,13 @@ class TreeVerifyStep:
         self.accept_len = torch.zeros(Bn, **i32)
         self.bonus = torch.zeros(Bn, **i32)
         self.kv_len_out = torch.zeros(Bn, **i32)
-        # workspaces (zero-filled once; the library leaves its counters at zero)
-        self.ws_expand = B.zeroed_workspace(max(B.adt_tree_expand_workspace_size(kmax, s.V, kmax), 16), dev)
-        self.ws_rerank = B.zeroed_workspace(max(B.adt_tree_rerank_workspace_size(s.candidates(b))
-                                                for b in range(Bn)), dev)
+        # workspaces (zero-filled once; the library leaves its counters at
+        # zero); one expand and one rerank workspace per image's draft chain
+        self.ws_expand = [B.zeroed_workspace(max(B.adt_tree_expand_workspace_size(kmax, s.V, kmax), 16), dev)
+                          for _ in range(Bn)]
+        self.ws_rerank = [B.zeroed_workspace(B.adt_tree_rerank_workspace_size(s.candidates(b)), dev)
+                          for b in range(Bn)]
+        self.draft_streams = [torch.cuda.Stream(device=dev) for _ in range(Bn)] if Bn > 1 else []
         self.ws_attn = B.zeroed_workspace(
             B.adt_tree_attn_workspace_size(Bn, s.H, s.D, s.max_nodes, self.lmax), dev)
 
@@ -131,32 +140,49 @@ class TreeVerifyStep:
                 self.root_token] + list(self.draft_rows)
 
     # -------------------------------------------------------------- phases
-    def launch_draft(self, stream=None):
-        """Expand d_b layers and rerank, for every image."""
+    def launch_draft_image(self, b, stream=None):
+        """Expand d_b layers and rerank, for image b."""
         s = self.shape
-        for b in range(s.batch):
-            k = s.width[b]
-            base = 0
-            fscore, fid = self.root_score, self.root_id
-            rows = self.draft_rows[b]
-            for d in range(s.depth[b]):
-                F = 1 if d == 0 else k
-                nxt = d % 2
-                B.adt_tree_expand(rows[d, :F], fscore, fid, F=F, V=s.V, k_child=k, k_keep=k,
-                                  temperature=1.0, child_id_base=base,
-                                  child_token=self.pool_tok[b][base:base + F * k],
-                                  child_logp=self.pool_logp[b][base:base + F * k],
-                                  child_score=self.pool_score[b][base:base + F * k],
-                                  child_parent=self.pool_par[b][base:base + F * k],
-                                  keep_idx=self.keep_idx[:k], next_score=self.front_score[nxt, :k],
-                                  next_id=self.front_id[nxt, :k], workspace=self.ws_expand, stream=stream)
-                fscore, fid = self.front_score[nxt, :k], self.front_id[nxt, :k]
-                base += F * k
-            lo, hi = int(self.node_offsets_host(b)), int(self.node_offsets_host(b + 1))
-            B.adt_tree_rerank(self.pool_tok[b], self.pool_score[b], self.pool_par[b], base,
-                              self.root_token[b:b + 1], hi - lo, tokens=self.tokens[lo:hi],
-                              parents=self.parents[lo:hi], cand_index=self.cand_index[lo:hi],
-                              depth=self.node_depth[lo:hi], workspace=self.ws_rerank, stream=stream)
+        k = s.width[b]
+        base = 0
+        fscore, fid = self.root_score, self.root_id
+        rows = self.draft_rows[b]
+        front_score, front_id, keep = self.front_score[b], self.front_id[b], self.keep_idx[b]
+        for d in range(s.depth[b]):
+            F = 1 if d == 0 else k
+            nxt = d % 2
+            B.adt_tree_expand(rows[d, :F], fscore, fid, F=F, V=s.V, k_child=k, k_keep=k,
+                              temperature=1.0, child_id_base=base,
+                              child_token=self.pool_tok[b][base:base + F * k],
+                              child_logp=self.pool_logp[b][base:base + F * k],
+                              child_score=self.pool_score[b][base:base + F * k],
+                              child_parent=self.pool_par[b][base:base + F * k],
+                              keep_idx=keep[:k], next_score=front_score[nxt, :k],
+                              next_id=front_id[nxt, :k], workspace=self.ws_expand[b], stream=stream)
+            fscore, fid = front_score[nxt, :k], front_id[nxt, :k]
+            base += F * k
+        lo, hi = int(self.node_offsets_host(b)), int(self.node_offsets_host(b + 1))
+        B.adt_tree_rerank(self.pool_tok[b], self.pool_score[b], self.pool_par[b], base,
+                          self.root_token[b:b + 1], hi - lo, tokens=self.tokens[lo:hi],
+                          parents=self.parents[lo:hi], cand_index=self.cand_index[lo:hi],
+                          depth=self.node_depth[lo:hi], workspace=self.ws_rerank[b], stream=stream)
+
+    def launch_draft(self, stream=None):
+        """Expand d_b layers and rerank, for every image: one chain, or with
+        several images one chain per image on its own stream, forked from
+        `stream` and joined back to it."""
+        if self.shape.batch == 1:
+            self.launch_draft_image(0, stream)
+            return
+        main = stream if stream is not None else torch.cuda.current_stream()
+        fork = torch.cuda.Event()
+        fork.record(main)
+        for b, sb in enumerate(self.draft_streams):
+            sb.wait_event(fork)
+            self.launch_draft_image(b, sb)
+            join = torch.cuda.Event()
+            join.record(sb)
+            main.wait_event(join)
 
     def node_offsets_host(self, i):
         return sum(self.n[:i])

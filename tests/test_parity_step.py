@@ -103,3 +103,46 @@ def test_step_llamagen_width_39_tree_of_256(mode, plant):
     a = _check(step, inp, tree, mode, layers=[0, 1])
     if mode == B.ACCEPT_GREEDY:
         assert a >= 2
+
+
+def test_ragged_batch_graph_replay_equals_eager():
+    """Eight images of different depth, width and prefix length: each image's
+    draft chain runs on its own stream, forked from the step's stream and
+    joined before attention.  The grown trees match the oracle; a captured
+    graph of the step, replayed over zeroed outputs, reproduces the eager
+    step bit for bit (trees, attention of every layer, acceptance, cache)."""
+    kv = [751, 1596, 1444, 640, 1427, 1245, 2352, 1248]
+    depth, width = [4, 7, 8, 7, 6, 6, 7, 6], [6, 8, 4, 2, 2, 1, 6, 4]
+    layers, H, D, V = 2, 8, 128, 16384
+    shape = StepShape(layers=layers, H=H, Hkv=H, D=D, V=V, kv_len=kv, depth=depth, width=width, max_nodes=64)
+    step = TreeVerifyStep(shape, keep_layer_outputs=True)
+    inp = synth.step_inputs(layers, H, H, D, V, kv, depth, width, step.n, step.lmax, 31)
+    step.load_inputs(inp)
+    B.adt_get_device_error()
+    step.launch()
+    torch.cuda.synchronize()
+    assert B.adt_get_device_error() == 0
+    trees = [draft_tree(inp["draft_rows"][b], width[b], depth[b], int(inp["root_token"][b]), step.n[b])
+             for b in range(len(kv))]
+    assert np.array_equal(step.tokens.cpu().numpy(), np.concatenate([t["tokens"] for t in trees]))
+    assert np.array_equal(step.parents.cpu().numpy(), np.concatenate([t["parents"] for t in trees]))
+    outs = ("tokens", "parents", "cand_index", "attn_out", "path", "accept_len", "bonus", "kv_len_out")
+    eager = {name: getattr(step, name).clone() for name in outs}
+    eager_k, eager_v = step.k_cache.clone(), step.v_cache.clone()
+
+    g = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(g, stream=s):
+            step.launch(s)
+    torch.cuda.synchronize()
+    for name in outs:
+        getattr(step, name).zero_()
+    with torch.cuda.stream(s):
+        g.replay()
+    torch.cuda.synchronize()
+    assert B.adt_get_device_error() == 0
+    for name in outs:
+        assert torch.equal(getattr(step, name), eager[name]), name
+    assert torch.equal(step.k_cache.view(torch.int16), eager_k.view(torch.int16))
+    assert torch.equal(step.v_cache.view(torch.int16), eager_v.view(torch.int16))
