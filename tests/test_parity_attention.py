@@ -96,6 +96,21 @@ def test_long_prefixes(sizes, kv, H, D):
     assert np.abs(lse - ref_lse).max() < LSE_ATOL
 
 
+@pytest.mark.parametrize("nb", [2, 32, 33])
+def test_tree_order_by_prefix_length(nb):
+    """Launches of 2-32 trees hand their slots to the trees by decreasing
+    prefix length (ties to the lower index); 33 trees keep tree order.
+    Prefix lengths repeat, so ties occur; every tree's output is checked."""
+    g = np.random.default_rng(nb)
+    kv = g.choice([0, 1, 63, 64, 65, 200, 200, 333], size=nb).tolist()
+    sizes = g.integers(1, 21, size=nb).tolist()
+    case = AttnCase(sizes, kv, 2, 2, 64, seed=700 + nb, lmax=max(kv) + 8)
+    got, lse, _ = case.run_gpu(max_nodes=max(sizes), max_kv=max(kv) + 8)
+    ref, ref_lse = case.run_oracle()
+    assert_attention_close(got, ref)
+    assert np.abs(lse - ref_lse).max() < LSE_ATOL
+
+
 def test_batch_of_eight_ragged_prefixes():
     g = np.random.default_rng(5)
     kv = g.integers(600, 2401, size=8).tolist()
