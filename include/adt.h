@@ -103,6 +103,18 @@ adt_status adt_get_device_error(void* stream, uint32_t* bits);
 /* Human-readable name of a status code (static string). */
 const char* adt_status_string(adt_status s);
 
+/* Testing hook, not for production use.  Every wait of adt_tree_attn's
+ * pipeline (a CTA waiting for its loads, products or softmax stages) is
+ * bounded: after `polls` unsuccessful polls it gives up, sets
+ * ADT_DEVERR_TIMEOUT in the device error word and the kernel leaves cleanly
+ * (the copies and tensor-core products it already issued are waited for
+ * first, so the device stays usable; the outputs of that call are
+ * unspecified).  This sets the bound for the launches that follow in this
+ * process; 0 restores the default (2^20 polls).  It lets a test make a
+ * bounded wait run out without any fault; it is not synchronised with
+ * calls on other threads. */
+adt_status adt_testing_set_wait_limit(uint32_t polls);
+
 /* ------------------------------------------------------------------------
  * adt_tree_attn - tree-masked attention for one transformer layer.
  *
@@ -147,18 +159,23 @@ adt_status adt_tree_attn(const adt_bf16* q, const adt_bf16* k_cache, const adt_b
  * every device allocation; a latency-critical thread that must not call
  * cudaMalloc, which may synchronise the device).  It computes what
  * adt_tree_attn computes, with the same arguments minus the workspace, and
- * allocates nothing: its scratch is one fixed 8 MiB array per device, held
+ * allocates nothing: its scratch is one fixed 4 MiB array per device, held
  * by every GPU that loads the library until the process exits.
  *   - The first call on each device looks up that array's device address;
  *     make this first call before any stream capture begins.
- *   - Every call shares the array (it keeps the last call's contents; the
- *     call clears what must start at zero on `stream` itself).  Calls that
- *     overlap on the GPU (other streams, other host threads) race on it:
- *     serialise them.
- *   - The key range is split into fewer pieces when the partial results of
- *     the usual split would not fit; a shape whose partials do not fit even
- *     unsplit (B * H * 64 * (D + 2) * 4 bytes plus tickets > 8 MiB) returns
- *     ADT_ERR_WORKSPACE and launches nothing.
+ *   - Only launches whose key splits merge through memory use the array:
+ *     more than 8 splits per (tree, query tile, head), which the split
+ *     heuristic picks when B * ceil(max_nodes/64) * H is small.  They take
+ *     B * ceil(max_nodes/64) * H * (4 + splits * 64 * (D + 2) * 4) bytes;
+ *     where that exceeds 4 MiB the key range is cut into fewer splits (at
+ *     most 8 of them merge on chip and need no scratch), so every shape
+ *     this call accepts fits.  Shapes beyond the limits of adt_tree_attn
+ *     (B * ceil(max_nodes/64) * H > 65536) return ADT_ERR_INVALID_ARG and
+ *     launch nothing.
+ *   - Every call shares the array, which keeps the last call's contents;
+ *     the call clears what must start at zero (its completion counters) on
+ *     `stream` itself.  Calls that overlap on the GPU (other streams, other
+ *     host threads) race on it: serialise them.
  * ------------------------------------------------------------------------ */
 adt_status adt_tree_attn_noalloc(const adt_bf16* q, const adt_bf16* k_cache,
                                  const adt_bf16* v_cache, const int32_t* kv_len,

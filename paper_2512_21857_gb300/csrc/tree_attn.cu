@@ -117,6 +117,7 @@ struct TcParams {
   float2* part_ml;    // [B][H][splits][64]
   unsigned* tickets;  // [B][H]
   unsigned* err;
+  uint32_t wait_limit;  // polls before a pipeline wait gives up (kWaitLimit unless a test lowers it)
 };
 
 // Byte offset of 16-byte chunk `ch` (0 .. D/8-1) of row `row` in a tile of
@@ -269,11 +270,13 @@ struct Barriers {
   uint64_t recv;                   // cluster merge: every split's rows for this owner landed
 };
 
-// Bounded wait that also gives up when another role has aborted.
+// Bounded wait of the pipeline that also gives up when another role has
+// aborted.  (The waits that let in-flight copies and products land before a
+// CTA leaves always keep the full kWaitLimit.)
 __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                         unsigned* err) {
+                                         unsigned* err, uint32_t limit) {
   const uint32_t a = sm100::smem_addr(bar);
-  for (uint32_t i = 0; i < kWaitLimit; ++i) {
+  for (uint32_t i = 0; i < limit; ++i) {
     if (sm100::mbar_try_wait(a, parity)) return true;
     if ((i & 255u) == 255u && *abort_flag) return false;
   }
@@ -578,27 +581,27 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int st = j % NS;
         // slot st was last used by chunk j - NS: its K is free once its S is
         // done, its V once its PV is done
-        if (!wait_bar(load_v ? &bars.done[st] : &bars.k_free[st], ((j / NS) - 1) & 1, &s_abort, p.err)) break;
+        if (!wait_bar(load_v ? &bars.done[st] : &bars.k_free[st], ((j / NS) - 1) & 1, &s_abort, p.err, p.wait_limit)) break;
         issue_tile(j);
         ++issued;
       }
-      if (s_abort) {
-        // let every copy still in flight land before the CTA can exit
-        for (int j = (issued > NS ? issued - NS : 0); j < issued; ++j)
-          (void)sm100::mbar_wait_bounded(sm100::smem_addr(load_v ? &bars.v_full[j % NS] : &bars.k_full[j % NS]),
-                                         (j / NS) & 1, kWaitLimit);
-      }
+      // Every copy issued lands before the CTA goes on: after an abort
+      // elsewhere its consumer may never have waited for it (on the normal
+      // path these waits return at once).
+      for (int j = (issued > NS ? issued - NS : 0); j < issued; ++j)
+        (void)sm100::mbar_wait_bounded(sm100::smem_addr(load_v ? &bars.v_full[j % NS] : &bars.k_full[j % NS]),
+                                       (j / NS) & 1, kWaitLimit);
     }
     __syncwarp();
   } else if (warp == kSMmaWarp) {
     // ------------------------------------------------------------ S = Q K^T
     if (lane == 0) {
-      bool ok = wait_bar(&bars.q_full, 0, &s_abort, p.err);
+      bool ok = wait_bar(&bars.q_full, 0, &s_abort, p.err, p.wait_limit);
       const uint32_t q_addr = sm100::smem_addr(sQ);
       for (int j = 0; ok && j < nch; ++j) {
         const int st = j % NS, sb = j & 1;
-        if (!wait_bar(&bars.k_full[st], (j / NS) & 1, &s_abort, p.err) ||
-            (j >= 2 && !wait_bar(&bars.s_free[sb], ((j >> 1) - 1) & 1, &s_abort, p.err)))
+        if (!wait_bar(&bars.k_full[st], (j / NS) & 1, &s_abort, p.err, p.wait_limit) ||
+            (j >= 2 && !wait_bar(&bars.s_free[sb], ((j >> 1) - 1) & 1, &s_abort, p.err, p.wait_limit)))
           break;
         sm100::tc_fence_after();
         const uint32_t k_addr = sm100::smem_addr(sStage + st * C::kStageBytes);
@@ -611,11 +614,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         sm100::mma_commit(sm100::smem_addr(&bars.s_full[sb]));
       }
-      if (s_abort) {
-        // wait for the tensor core to finish whatever was issued
-        sm100::mma_commit(sm100::smem_addr(&bars.drain[0]));
-        (void)sm100::mbar_wait_bounded(sm100::smem_addr(&bars.drain[0]), 0, kWaitLimit);
-      }
+      // The tensor core finishes whatever was issued before this thread goes
+      // on, also when a consumer aborted after the last product was issued.
+      sm100::mma_commit(sm100::smem_addr(&bars.drain[0]));
+      (void)sm100::mbar_wait_bounded(sm100::smem_addr(&bars.drain[0]), 0, kWaitLimit);
     }
     __syncwarp();
   } else if (warp == kPvMmaWarp) {
@@ -626,8 +628,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       // every k step.
       const uint64_t ones_desc = sm100::smem_desc_sw128(sm100::smem_addr(smem + C::kOnesOff), C::kBlock128, 1024);
       for (int i = 0; i < nch; ++i) {
-        if (!wait_bar(&bars.p_full[i & 1], (i >> 1) & 1, &s_abort, p.err) ||
-            !wait_bar(&bars.v_full[i % NS], (i / NS) & 1, &s_abort, p.err))
+        if (!wait_bar(&bars.p_full[i & 1], (i >> 1) & 1, &s_abort, p.err, p.wait_limit) ||
+            !wait_bar(&bars.v_full[i % NS], (i / NS) & 1, &s_abort, p.err, p.wait_limit))
           break;
         sm100::tc_fence_after();
         const uint32_t v_addr = sm100::smem_addr(sStage + (i % NS) * C::kStageBytes + C::kStageTile);
@@ -642,10 +644,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         sm100::mma_commit(sm100::smem_addr(&bars.done[i % NS]));
       }
-      if (s_abort) {
-        sm100::mma_commit(sm100::smem_addr(&bars.drain[1]));
-        (void)sm100::mbar_wait_bounded(sm100::smem_addr(&bars.drain[1]), 0, kWaitLimit);
-      }
+      sm100::mma_commit(sm100::smem_addr(&bars.drain[1]));
+      (void)sm100::mbar_wait_bounded(sm100::smem_addr(&bars.drain[1]), 0, kWaitLimit);
     }
     __syncwarp();
   } else {
@@ -670,7 +670,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     float mua = -INFINITY, mub = -INFINITY;  // running maxima used for the exponentials
     for (int j = 0; j < nch; ++j) {
       const int sb = j & 1;
-      if (!__all_sync(adt::kFullMask, wait_bar(&bars.s_full[sb], (j >> 1) & 1, &s_abort, p.err))) break;
+      if (!__all_sync(adt::kFullMask, wait_bar(&bars.s_full[sb], (j >> 1) & 1, &s_abort, p.err, p.wait_limit))) break;
       // S(j) is complete, so its K tile can be refilled (the S issuer goes
       // straight on to the next S product).
       if (warp == 0 && lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.k_free[j % NS]));
@@ -729,7 +729,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
       // P buffer sb was last read by the PV product of chunk j - 2.
       if (j >= 2 && !__all_sync(adt::kFullMask,
-                                wait_bar(&bars.done[(j - 2) % NS], ((j - 2) / NS) & 1, &s_abort, p.err)))
+                                wait_bar(&bars.done[(j - 2) % NS], ((j - 2) / NS) & 1, &s_abort, p.err, p.wait_limit)))
         break;
       {
         const uint32_t pbase = sm100::smem_addr(sP) + sb * C::kPBytes + st_row * 128;
@@ -746,7 +746,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // Cache rows at or past L in this chunk (the end of the prefix) can
       // hold anything, NaN included, and P is 0 there: zero their V rows.
       if (!tree_j && kl < keys) {
-        if (!__all_sync(adt::kFullMask, wait_bar(&bars.v_full[j % NS], (j / NS) & 1, &s_abort, p.err))) break;
+        if (!__all_sync(adt::kFullMask, wait_bar(&bars.v_full[j % NS], (j / NS) & 1, &s_abort, p.err, p.wait_limit))) break;
         uint8_t* vt = sStage + (j % NS) * C::kStageBytes + C::kStageTile;
         const int per_row = C::kBlocks * 8;
         for (int i = tid; i < (keys - kl) * per_row; i += kSoftmaxWarps * 32) {
@@ -759,7 +759,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // Raise O to the new maxima (rare): needs the previous PV product done.
       if (j > 0 && __any_sync(adt::kFullMask, alpha_a != 1.f || alpha_b != 1.f)) {
         if (!__all_sync(adt::kFullMask,
-                        wait_bar(&bars.done[(j - 1) % NS], ((j - 1) / NS) & 1, &s_abort, p.err)))
+                        wait_bar(&bars.done[(j - 1) % NS], ((j - 1) / NS) & 1, &s_abort, p.err, p.wait_limit)))
           break;
         sm100::tc_fence_after();
 #pragma unroll 1
@@ -807,7 +807,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int last = nch - 1;
     // s_abort can change under the warp: decide once, by a vote.
     if (__all_sync(adt::kFullMask, nch > 0 && !s_abort))
-      have_o = __all_sync(adt::kFullMask, wait_bar(&bars.done[last % NS], (last / NS) & 1, &s_abort, p.err));
+      have_o = __all_sync(adt::kFullMask, wait_bar(&bars.done[last % NS], (last / NS) & 1, &s_abort, p.err, p.wait_limit));
     if (have_o) {
       sm100::tc_fence_after();
       const uint32_t lane_base = static_cast<uint32_t>(warp * 32) << 16;
@@ -1209,6 +1209,10 @@ adt_status check_args(const adt_bf16* q, const adt_bf16* k_cache, const adt_bf16
   return ADT_OK;
 }
 
+// Polls before a pipeline wait gives up; 0 = kWaitLimit.  Set only by
+// adt_testing_set_wait_limit.
+uint32_t g_wait_limit = 0;
+
 TcParams make_params(const adt_bf16* q, const int32_t* kv_len, const adt_bf16* k_tree, const adt_bf16* v_tree,
                      const int32_t* parents, const int32_t* node_offsets, int B, int H, int Hkv, int max_kv,
                      int max_nodes, int splits, float scale, adt_bf16* out, float* lse, unsigned* err) {
@@ -1230,12 +1234,19 @@ TcParams make_params(const adt_bf16* q, const int32_t* kv_len, const adt_bf16* k
   prm.out = reinterpret_cast<__nv_bfloat16*>(out);
   prm.lse = lse;
   prm.err = err;
+  const uint32_t lim = __atomic_load_n(&g_wait_limit, __ATOMIC_RELAXED);
+  prm.wait_limit = lim ? lim : kWaitLimit;
   return prm;
 }
 
 }  // namespace
 
 extern "C" {
+
+adt_status adt_testing_set_wait_limit(uint32_t polls) {
+  __atomic_store_n(&g_wait_limit, polls, __ATOMIC_RELAXED);
+  return ADT_OK;
+}
 
 size_t adt_tree_attn_workspace_size(int32_t B, int32_t H, int32_t D, int32_t max_nodes,
                                     int32_t max_kv) {
@@ -1286,10 +1297,10 @@ adt_status adt_tree_attn(const adt_bf16* q, const adt_bf16* k_cache, const adt_b
 // array instead.
 // ---------------------------------------------------------------------------
 
-// 8 MiB of scratch, held by every GPU that loads the library until the
+// 4 MiB of scratch, held by every GPU that loads the library until the
 // process exits.  Shared by all calls on a device: calls that overlap on the
 // GPU (different streams, or different host threads) race on it.
-static constexpr size_t kNoAllocScratchBytes = size_t(8) << 20;
+static constexpr size_t kNoAllocScratchBytes = size_t(4) << 20;
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 namespace {
@@ -1307,19 +1318,39 @@ void noalloc_setup(int dev) {
   g_noalloc_ptr[dev] = p;
 }
 
+// What a launch with `splits` key splits uses: nothing when the splits merge
+// inside their cluster (splits <= kMaxClusterSplits, the kernel returns
+// before it touches tickets or partials); otherwise Bq*H tickets, then
+// Bq*H*splits partial rows (m, l) and partial outputs of 64 rows x D.
 struct NoAllocLayout {
   size_t tickets, part_ml, part_o, total;
 };
 
-NoAllocLayout noalloc_layout(int B, int H, int D, int splits) {
+NoAllocLayout noalloc_layout(int Bq, int H, int D, int splits) {
   NoAllocLayout w{};
-  const size_t bh = static_cast<size_t>(B) * H;
+  if (splits <= kMaxClusterSplits) return w;
+  const size_t bh = static_cast<size_t>(Bq) * H;
   const size_t bhs = bh * splits;
   w.tickets = 0;
   w.part_ml = adt::align_up(bh * sizeof(unsigned), 256);
   w.part_o = adt::align_up(w.part_ml + bhs * kMaxNodes * sizeof(float2), 256);
   w.total = adt::align_up(w.part_o + bhs * kMaxNodes * D * sizeof(float), 256);
   return w;
+}
+
+// The split count of a no-allocation launch: the usual heuristic's, lowered
+// while a workspace merge's partials would not fit the scratch; once it is
+// down to a cluster's size the splits merge in their cluster and need no
+// scratch, and the count is lowered further until all clusters are
+// co-resident, as the heuristic does for its own cluster-sized counts.
+int noalloc_splits(int sm_count, int Bq, int H, int D, int max_kv, int dev, bool large) {
+  int s = choose_splits(sm_count, Bq, H, D, max_kv, dev, large);
+  while (s > kMaxClusterSplits && noalloc_layout(Bq, H, D, s).total > kNoAllocScratchBytes) --s;
+  if (s <= kMaxClusterSplits) {
+    const int bh = Bq * H;
+    while (s > 1 && max_active_clusters(D, large, s, dev) < bh) --s;
+  }
+  return s;
 }
 
 }  // namespace
@@ -1342,17 +1373,20 @@ extern "C" adt_status adt_tree_attn_noalloc(const adt_bf16* q, const adt_bf16* k
   if (info.device < 0 || info.device >= kNoAllocMaxDevices) return ADT_ERR_UNSUPPORTED;
   std::call_once(g_noalloc_once[info.device], noalloc_setup, info.device);
   if (g_noalloc_status[info.device] != cudaSuccess || !g_noalloc_ptr[info.device]) return ADT_ERR_CUDA;
-  // As many splits as the usual heuristic picks, fewer if the partials would
-  // not fit; a shape that does not fit even unsplit is rejected.
   const int Bq = B * qtiles_for(max_nodes);
-  int splits = choose_splits(info.sm_count, Bq, H, D, max_kv, info.device, max_nodes > kMaxNodes);
-  while (splits > 1 && noalloc_layout(Bq, H, D, splits).total > kNoAllocScratchBytes) --splits;
+  const int splits = noalloc_splits(info.sm_count, Bq, H, D, max_kv, info.device, max_nodes > kMaxNodes);
   const NoAllocLayout w = noalloc_layout(Bq, H, D, splits);
+  // Unreachable for the shapes check_args accepts (a workspace merge is
+  // chosen only when its partials fit); kept as the guard of the array.
   if (w.total > kNoAllocScratchBytes) return ADT_ERR_WORKSPACE;
   uint8_t* ws = static_cast<uint8_t*>(g_noalloc_ptr[info.device]);
   cudaStream_t s = adt::as_stream(stream);
-  // The array keeps the previous call's contents: the tickets must start at zero.
-  ADT_CUDA_TRY(cudaMemsetAsync(ws + w.tickets, 0, static_cast<size_t>(Bq) * H * sizeof(unsigned), s));
+  // A workspace merge counts finished splits in tickets that start at zero.
+  // A completed call leaves them at zero, but one that a bounded wait ended
+  // (ADT_DEVERR_TIMEOUT) can leave them set, so they are cleared here, on
+  // the caller's stream.  Cluster merges use no tickets.
+  if (splits > kMaxClusterSplits)
+    ADT_CUDA_TRY(cudaMemsetAsync(ws + w.tickets, 0, static_cast<size_t>(Bq) * H * sizeof(unsigned), s));
   TcParams prm = make_params(q, kv_len, k_tree, v_tree, parents, node_offsets, B, H, Hkv, max_kv, max_nodes, splits,
                              softmax_scale, out, lse, info.error_word);
   prm.part_o = reinterpret_cast<float*>(ws + w.part_o);
