@@ -121,6 +121,21 @@ def test_batch_of_eight_ragged_prefixes():
     assert_attention_close(got, ref)
 
 
+def test_ragged_batch_bench_launch():
+    """The launch the ragged 8-image benchmark times, at its exact shape: 8
+    trees (the sizes its depths and widths give), 32 heads x 128, its prefix
+    lengths.  256 (tree, head) pairs take one split each (256 CTAs on the
+    GPU's SMs, no merge) and the launch slots go to the trees longest prefix
+    first."""
+    kv = [751, 1596, 1444, 640, 1427, 1245, 2352, 1248]
+    sizes = [64, 64, 64, 27, 23, 7, 64, 64]
+    case = AttnCase(sizes, kv, 32, 32, 128, seed=88, max_depth=10, max_children=8, lmax=2352 + 64)
+    got, lse, _ = case.run_gpu(max_nodes=64, max_kv=2352 + 64)
+    ref, ref_lse = case.run_oracle()
+    assert_attention_close(got, ref)
+    assert np.abs(lse - ref_lse).max() < LSE_ATOL
+
+
 def test_workspace_reuse_and_repeat_is_deterministic():
     case = AttnCase([26], [512], 8, 8, 64, seed=3)
     a, la, ws = case.run_gpu()
