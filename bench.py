@@ -222,10 +222,13 @@ def run_gpu(args, wl, rank, world):
         torch.distributed.barrier()
     torch.cuda.synchronize()
     t0 = time.time()
+    step_ev = [torch.cuda.Event(enable_timing=True) for _ in range(K + 1)]
     with torch.cuda.stream(stream):
         ev0.record(stream)
-        for _ in range(K):
+        step_ev[0].record(stream)
+        for i in range(K):
             step_graph.replay()
+            step_ev[i + 1].record(stream)
         ev1.record(stream)
         ea0.record(stream)
         for _ in range(K):
@@ -237,6 +240,8 @@ def run_gpu(args, wl, rank, world):
         torch.distributed.barrier()
     clocks = sampler.stop(t0, t1)
     step_ms = ev0.elapsed_time(ev1) / K
+    per_step = sorted(step_ev[i].elapsed_time(step_ev[i + 1]) for i in range(K))
+    pct = {f"p{q}": per_step[min(K - 1, int(round(q / 100 * (K - 1))))] for q in (10, 50, 90)}
     attn_ms = ea0.elapsed_time(ea1) / (K * shape.layers)
     errbits = B.adt_get_device_error(stream)
     if errbits:
@@ -317,7 +322,7 @@ def run_gpu(args, wl, rank, world):
     achieved = ab["attention_per_layer"] / (attn_ms * 1e-3) / 1e9
     sha = attn_source_sha()
     traffic = NCU_TRAFFIC.get(sha) if args.workload == "7b" else None
-    return dict(step_ms=step_ms, attn_ms=attn_ms, clocks=clocks, e2e_ms=e2e_ms, h2d=h2d, d2h=d2h,
+    return dict(step_ms=step_ms, step_pct=pct, attn_ms=attn_ms, clocks=clocks, e2e_ms=e2e_ms, h2d=h2d, d2h=d2h,
                 launches=K * (step.kernel_launches_per_step() + shape.layers), achieved=achieved, peak=peak, peak_kind=peak_kind,
                 traffic=traffic, attn_bytes=ab["attention_per_layer"], step_bytes=ab["attention"], sha=sha)
 
@@ -377,7 +382,7 @@ class OracleSample:
 
         wl = self.wl
         L, D, n, k = wl["kv_len"][self.image], wl["D"], self.n, wl["width"][self.image]
-        t = time.perf_counter()
+        t = t_start = time.perf_counter()
         nq = self.nq
         for _ in range(self.layers_sampled):
             oracle.tree_attention(self.q[:nq], self.kc, self.vc, [L], self.kt[:nq], self.vt[:nq],
@@ -394,16 +399,55 @@ class OracleSample:
         t = time.perf_counter()
         oracle.kv_compact(self.kc16, self.kc16, [L], self.kt16, self.kt16, [0, n], [[0, 1]])
         t_cmp = (time.perf_counter() - t) * wl["layers"]
+        self.wall = time.perf_counter() - t_start   # the seconds actually spent
+        self.parts = dict(attn=t_attn, expand=t_exp, accept=t_acc, commit=t_cmp)
         return t_attn + t_exp + t_acc + t_cmp
 
+    def run_attention_only(self):
+        """One sampled layer of attention for this sample's heads (seconds)."""
+        wl = self.wl
+        nq = self.nq
+        t = time.perf_counter()
+        oracle_mod().tree_attention(self.q[:nq], self.kc, self.vc, [wl["kv_len"][self.image]], self.kt[:nq],
+                                    self.vt[:nq], self.tb.parents[:nq], [0, nq], 1.0 / math.sqrt(wl["D"]))
+        return time.perf_counter() - t
 
-def cpu_sample_subprocess(wl_key, heads, layers_sampled, rows_sampled, reps, nodes=0):
-    """Runs oracle samples in a fresh single-threaded process."""
+
+def oracle_mod():
+    import oracle
+    return oracle
+
+
+def _attention_worker(job):
+    """All-core leg: one worker process builds a sample of `heads` heads and
+    times one layer of the oracle's attention for them (single-threaded)."""
+    wl_key, seed, heads, image = job
+    smp = OracleSample(WORKLOADS[wl_key], seed, heads, 1, 1, image=image)
+    smp.run_attention_only()  # first touch of the inputs, untimed
+    return smp.run_attention_only()
+
+
+def cpu_model():
+    """The host CPU's model name (lscpu), for the record."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
+def cpu_sample_subprocess(wl_key, heads, layers_sampled, rows_sampled, reps, nodes=0, procs=1):
+    """Runs oracle samples in a fresh single-threaded process (and, with
+    procs > 1, the all-core attention leg in a pool of that many)."""
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
                CUDA_VISIBLE_DEVICES="")
     cmd = [sys.executable, os.path.abspath(__file__), "--cpu-sample", wl_key, "--cpu-heads", str(heads),
            "--cpu-layers", str(layers_sampled), "--cpu-rows", str(rows_sampled), "--cpu-reps", str(reps),
-           "--cpu-nodes", str(nodes)]
+           "--cpu-nodes", str(nodes), "--cpu-procs", str(procs)]
     out = subprocess.run(cmd, capture_output=True, text=True, env=env, timeout=1800)
     if out.returncode != 0:
         raise RuntimeError(out.stderr[-2000:])
@@ -415,11 +459,41 @@ def cpu_sample_main(args):
     samples = [OracleSample(wl, 7 + b, args.cpu_heads, args.cpu_layers, args.cpu_rows, image=b,
                             nodes_sampled=args.cpu_nodes)
                for b in range(len(wl["kv_len"]))]
-    times = [sum(smp.run() for smp in samples) for _ in range(args.cpu_reps)]
+    times, wall = [], 0.0
+    for _ in range(args.cpu_reps):
+        times.append(sum(smp.run() for smp in samples))
+        wall += sum(smp.wall for smp in samples)
     desc = samples[0].desc
     if len(samples) > 1:
         desc = f"per image of the {len(samples)}, summed: " + desc
-    print(json.dumps({"sec_per_step": times, "desc": desc}))
+    res = {"sec_per_step": times, "desc": desc, "sampled_wall_s": wall,
+           "parts": {k: sum(smp.parts[k] for smp in samples) for k in samples[0].parts}}
+    if args.cpu_procs > 1 and len(samples) == 1:
+        # All cores: the attention sample (every head of one layer) split over
+        # worker processes, one thread each, running concurrently; the step
+        # time is their slowest worker x layers plus the other parts as timed
+        # on one core.
+        import multiprocessing as mp
+        wl_h = wl["H"]
+        P = min(args.cpu_procs, wl_h)
+        per = [wl_h // P + (1 if i < wl_h % P else 0) for i in range(P)]
+        ctx = mp.get_context("spawn")
+        with ctx.Pool(P) as pool:
+            pool.map(_attention_worker, [(args.cpu_sample, 7, 1, 0)] * P)  # start-up, imports
+            walls = []
+            for _ in range(args.cpu_reps):
+                t0 = time.perf_counter()
+                w = pool.map(_attention_worker, [(args.cpu_sample, 7, h, 0) for h in per], chunksize=1)
+                walls.append((max(w), time.perf_counter() - t0))
+        attn_layer = statistics.median(x[0] for x in walls)
+        rest = samples[0].parts["expand"] + samples[0].parts["accept"] + samples[0].parts["commit"]
+        res["all_core"] = {"procs": P, "attn_layer_s": attn_layer,
+                           "sec_per_step": attn_layer * wl["layers"] + rest,
+                           "desc": f"oracle attention of all {wl_h} heads of one layer split over {P} worker "
+                                   f"processes (1 thread each, concurrent; the slowest worker's time) x "
+                                   f"{wl['layers']} layers, plus expansion, rerank, walk and commit as timed "
+                                   f"on one core; extrapolated to one full step"}
+    print(json.dumps(res))
 
 
 # ------------------------------------------------------------------ main
@@ -446,8 +520,9 @@ def run_decode(args):
     out, st = dec.generate(prompt)
     n = g * g
     t0 = time.perf_counter()
+    # vanilla greedy decoding in plain torch (bf16 scaled_dot_product_attention, no library call)
     ref, margins = greedy_decode(shape, dec.target_w, prompt, n, batch=args.decode_batch, return_margins=True,
-                                 graphs=graphs)
+                                 graphs=graphs, attn_dtype=torch.bfloat16)
     torch.cuda.synchronize()
     t_van = time.perf_counter() - t0
     same = sum(1 for b in range(args.decode_batch) for x, y in zip(out[b], ref[b]) if x == y)
@@ -488,6 +563,7 @@ def main():
     ap.add_argument("--cpu-rows", type=int, default=1)
     ap.add_argument("--cpu-reps", type=int, default=1)
     ap.add_argument("--cpu-nodes", type=int, default=0)
+    ap.add_argument("--cpu-procs", type=int, default=1)
     ap.add_argument("--decode", action="store_true", help="the end-to-end synthetic decode loop instead")
     ap.add_argument("--decode-batch", type=int, default=1)
     ap.add_argument("--decode-grid", type=int, default=48)
@@ -538,7 +614,9 @@ def main():
                 "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": config,
                 "cpu_baseline": {"kind": "oracle", "cores": 1, "sample": res["desc"], "value": value,
-                                 "unit": "steps/s"},
+                                 "unit": "steps/s", "extrapolated": True,
+                                 "sampled_wall_s": res["sampled_wall_s"], "cpu_model": cpu_model()},
+                "extrapolated": True,
                 "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
                 "wall_s": time.time() - t_run}
         print(json.dumps(line), flush=True)
@@ -558,15 +636,22 @@ def main():
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         if one:
-            res = cpu_sample_subprocess(args.workload, wl["H"], 1, 41, 5)
+            res = cpu_sample_subprocess(args.workload, wl["H"], 1, 41, 5, procs=min(os.cpu_count() or 1, 64))
         else:  # a bounded sample: 4 heads of one layer per image
             res = cpu_sample_subprocess(args.workload, 4, 1, 8, 3)
         sec = statistics.median(res["sec_per_step"])
-        cpu = {"value": 1.0 / sec, "unit": "steps/s", "cores": 1, "kind": "oracle", "sample": res["desc"]}
+        cpu = {"value": 1.0 / sec, "unit": "steps/s", "cores": 1, "kind": "oracle", "sample": res["desc"],
+               "extrapolated": True, "sampled_wall_s": res["sampled_wall_s"], "cpu_model": cpu_model(),
+               "host_cpus": os.cpu_count()}
+        if "all_core" in res:
+            ac = res["all_core"]
+            cpu["all_core"] = {"value": 1.0 / ac["sec_per_step"], "unit": "steps/s", "cores": ac["procs"],
+                               "sample": ac["desc"], "extrapolated": True}
     line = {
         "metric": metric, "value": value, "unit": "steps/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": r["step_ms"], "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": config,
+        "ms_per_step_percentiles": r["step_pct"],
         "hbm_gbs_step": r["step_bytes"] / (r["step_ms"] * 1e-3) / 1e9,
         "roofline": {"bound": "hbm", "kernel": "tree_attn_tc_kernel<128>" if wl["D"] == 128 else "tree_attn_tc_kernel<64>",
                      "achieved": r["achieved"], "peak": r["peak"], "unit": "GB/s",
