@@ -443,47 +443,121 @@ class Decoder:
 
 
 
+class DenseModel:
+    """The same decoder stack as TreeModel for vanilla decoding, without the
+    library: a plain KV cache tensor written by indexing, and attention by
+    torch's scaled_dot_product_attention (in fp32 by default) over the cache
+    with a causal mask.  Every image holds the same number of tokens (they
+    advance in lockstep), so one start position serves the batch.  The
+    shapes are static (attention always spans the whole cache, masked), so
+    a step can be captured in a CUDA graph."""
+
+    def __init__(self, shape: ModelShape, weights: DecoderWeights, batch: int, lmax: int, device,
+                 attn_dtype=torch.float32):
+        s = self.s = shape
+        self.w = weights
+        self.lmax = lmax
+        self.batch = batch
+        self.attn_dtype = attn_dtype
+        L = len(weights.layers)
+        bf = dict(dtype=torch.bfloat16, device=device)
+        self.k_cache = torch.zeros((L, batch, s.kv_heads, lmax, s.head_dim), **bf)
+        self.v_cache = torch.zeros((L, batch, s.kv_heads, lmax, s.head_dim), **bf)
+        self.keys = torch.arange(lmax, device=device)
+        self.device = device
+
+    def forward(self, x, start):
+        """x [batch, n, hidden]: n new tokens per image at positions start ..
+        start + n - 1 (start: a 0-d int64 device tensor).  Writes their K/V
+        into the cache and returns the final hidden states [batch, n, hidden]."""
+        s = self.s
+        Bn, n, _ = x.shape
+        hq, hk = s.heads * s.head_dim, s.kv_heads * s.head_dim
+        pos = start + torch.arange(n, device=self.device)
+        rows = pos.repeat(Bn)
+        visible = self.keys[None, :] <= pos[:, None]          # [n, lmax]: causal over the cache
+        group = s.heads // s.kv_heads
+        for li, lw in enumerate(self.w.layers):
+            h = _rms_norm(x, lw["ln1"], s.eps).view(Bn * n, -1)
+            qkv = h @ lw["wqkv"]
+            q = _rope(qkv[:, :hq].view(Bn * n, s.heads, s.head_dim), rows, s.rope_theta).to(torch.bfloat16)
+            k = _rope(qkv[:, hq:hq + hk].view(Bn * n, s.kv_heads, s.head_dim), rows, s.rope_theta).to(torch.bfloat16)
+            v = qkv[:, hq + hk:].view(Bn * n, s.kv_heads, s.head_dim).to(torch.bfloat16)
+            self.k_cache[li].index_copy_(2, pos, k.view(Bn, n, s.kv_heads, s.head_dim).transpose(1, 2))
+            self.v_cache[li].index_copy_(2, pos, v.view(Bn, n, s.kv_heads, s.head_dim).transpose(1, 2))
+            kc = self.k_cache[li].to(self.attn_dtype)
+            vc = self.v_cache[li].to(self.attn_dtype)
+            if group > 1:
+                kc = kc.repeat_interleave(group, dim=1)
+                vc = vc.repeat_interleave(group, dim=1)
+            qh = q.view(Bn, n, s.heads, s.head_dim).transpose(1, 2).to(self.attn_dtype)
+            o = torch.nn.functional.scaled_dot_product_attention(qh, kc, vc, attn_mask=visible,
+                                                                 scale=s.head_dim ** -0.5)
+            o = o.transpose(1, 2).reshape(Bn * n, hq).to(torch.bfloat16)
+            xf = x.view(Bn * n, -1) + o.to(x.dtype) @ lw["wo"]
+            h = _rms_norm(xf, lw["ln2"], s.eps)
+            gu = h @ lw["wgu"]
+            xf = xf + (torch.nn.functional.silu(gu[:, : s.ffn].float()) * gu[:, s.ffn:].float()).to(x.dtype) @ lw["wd"]
+            x = xf.view(Bn, n, -1)
+        return x
+
+
 def greedy_decode(shape: ModelShape, weights: DecoderWeights, prompt, n_tokens, device="cuda", batch=1,
-                  return_margins=False, graphs=False):
-    """Vanilla greedy decoding with the same target: one node per step (a
-    tree of its root alone).  Returns the tokens (and, with return_margins,
-    the top-1 minus top-2 logit gap of every decision over the standard
-    deviation of that logit row)."""
+                  return_margins=False, graphs=False, attn_dtype=torch.float32, forced=None):
+    """Vanilla greedy decoding with the same target, one token per step,
+    through DenseModel: none of the library's entry points (neither its
+    attention nor its KV commit) is on this path, so it is an independent
+    reference for the tree decoder's output (greedy verification is
+    lossless).  Returns the tokens (and, with return_margins, the top-1
+    minus top-2 logit gap of every decision over the standard deviation of
+    that logit row).  With graphs, each step replays one CUDA graph.
+
+    forced (a [batch][n_tokens] token list) teacher-forces the sequence: step
+    i still returns the target's greedy choice, but the token fed to step
+    i + 1 is forced[b][i], so every position of another decoder's output can
+    be checked against the target's choice given that output's own prefix."""
     if not 2 <= len(prompt) <= 257:
-        raise ValueError("prompt of 2 .. 257 tokens (the prefill is one tree)")
-    model = TreeModel(shape, weights, batch, len(prompt) + n_tokens + 16, len(prompt) - 1, device)
-    model.graphs_enabled = graphs
-    dev = device
+        raise ValueError("prompt of 2 .. 257 tokens")
     P = len(prompt)
-    n = P - 1
-    i32 = dict(dtype=torch.int32, device=dev)
-    tok = torch.tensor(list(prompt[:-1]) * batch, **i32)
-    par = torch.cat([_chain(n, dev)] * batch)
-    offs = torch.tensor([b * n for b in range(batch + 1)], **i32)
-    kv = torch.zeros(batch, **i32)
-    pos = torch.arange(n, device=dev, dtype=torch.int32).repeat(batch)
-    _, kt, vt = model.run(weights.embed[tok.long()], pos, par, offs, kv, batch)
-    path = torch.arange(n, **i32).repeat(batch, 1).contiguous()
-    kv_out = torch.empty(batch, **i32)
-    model.commit(kt, vt, kv, kv_out, offs, path, n, torch.full((batch,), n - 1, **i32), batch)
-    kv = kv_out.clone()
-    root = torch.full((batch,), int(prompt[-1]), **i32)
-    out, margins = [], []
-    one = torch.arange(batch + 1, **i32)
-    rootpar = torch.full((batch,), -1, **i32)
-    zpath = torch.zeros((batch, 1), **i32)
-    zlen = torch.zeros(batch, **i32)
-    for _ in range(n_tokens):
-        h, kt, vt = model.run(weights.embed[root.long()], kv, rootpar, one, kv, batch)
-        logits = lm_logits(weights, h, shape.eps)
+    model = DenseModel(shape, weights, batch, P + n_tokens + 16, device, attn_dtype)
+    dev = device
+    tok = torch.tensor(list(prompt[:-1]), dtype=torch.long, device=dev)
+    model.forward(weights.embed[tok][None].expand(batch, -1, -1).contiguous(),
+                  torch.zeros((), dtype=torch.long, device=dev))
+    start = torch.full((), P - 1, dtype=torch.long, device=dev)
+    root = torch.full((batch,), int(prompt[-1]), dtype=torch.long, device=dev)
+
+    def one_step():
+        h = model.forward(weights.embed[root][:, None, :], start)
+        logits = lm_logits(weights, h[:, 0], shape.eps)
         top2 = torch.topk(logits, 2, dim=-1)
-        nxt = top2.indices[:, 0].to(torch.int32)
-        model.commit(kt, vt, kv, kv_out, one, zpath, 1, zlen, batch)
-        kv = kv_out.clone()
+        return top2.indices[:, 0], (top2.values[:, 0] - top2.values[:, 1]) / logits.std(dim=-1)
+
+    graph = None
+    if graphs:
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        saved = [model.k_cache.clone(), model.v_cache.clone()]
+        with torch.cuda.stream(side):
+            one_step()  # warm-up outside the capture (it writes a cache row that is restored below)
+        torch.cuda.current_stream().wait_stream(side)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            g_next, g_margin = one_step()
+        model.k_cache.copy_(saved[0])
+        model.v_cache.copy_(saved[1])
+    feed = None if forced is None else torch.tensor(forced, dtype=torch.long, device=dev)
+    out, margins = [], []
+    for i in range(n_tokens):
+        if graph is not None:
+            graph.replay()
+            nxt, margin = g_next.clone(), g_margin.clone()
+        else:
+            nxt, margin = one_step()
         out.append(nxt)
-        if return_margins:
-            margins.append((top2.values[:, 0] - top2.values[:, 1]) / logits.std(dim=-1))
-        root = nxt
+        margins.append(margin)
+        root.copy_(nxt if feed is None else feed[:, i])
+        start += 1
     toks = torch.stack(out, 1).cpu().tolist()
     if return_margins:
         return toks, torch.stack(margins, 1).cpu().tolist()

@@ -1,12 +1,23 @@
 """The end-to-end decode loop (random-init target, EAGLE-style draft head,
 ADT-Tree trees every step) against vanilla greedy decoding with the same
-target: greedy verification is lossless, so both must emit the same tokens.
-The two run different launch shapes (a tree of up to 64 nodes vs one node,
-batched GEMMs of different sizes), so their logits agree only to rounding;
-a difference is allowed only where vanilla decoding itself faced a near tie
-(top-2 logit gap below 1 % of the logit row's standard deviation: a bf16
-residual stream moves logits of spread s by about s / 2^8 between the two
-shapes), and the comparison stops there."""
+target weights: greedy verification is lossless (Sec. 5.1 / 5.2: acceptance
+is not relaxed, so the output is the target's own), so both must emit the
+same tokens.  The reference decodes one token per step in plain torch: its
+own KV cache tensor and fp32 scaled_dot_product_attention, none of the
+library's entry points, so a fault shared by the library's attention or KV
+commit cannot cancel out.  It is teacher-forced with the tree decoder's
+output, so every emitted token is checked: it must be the target's greedy
+choice given the tokens before it.  The two paths round differently (bf16
+probabilities in the library's P.V product, batched GEMMs of different
+shapes), so their logits agree only to rounding; a token may differ from
+the reference's choice only where the reference itself faced a near tie
+(a top-2 logit gap below a bound relative to the logit row's standard
+deviation), and such positions must be rare.  The bound follows from how
+far the two paths' hidden states drift apart: with a bf16 residual stream
+they differ by about 0.7 % after two layers (different GEMM shapes round
+differently), which moves a top-2 gap by about sqrt(2) x 0.7 % ~ 1 % of the
+row's spread per standard deviation, so 3 % covers three; with an fp32
+stream only the attention's bf16 arithmetic differs, and 1 % is kept."""
 import pytest
 import torch
 
@@ -15,7 +26,8 @@ from paper_2512_21857_gb300 import binding as B
 from paper_2512_21857_gb300.decode import Decoder, DecoderWeights, ModelShape, greedy_decode
 
 pytestmark = pytest.mark.gpu
-NEAR_TIE = 0.01  # of the logit row's standard deviation
+NEAR_TIE_BF16 = 0.03  # of the logit row's standard deviation, bf16 residual stream
+NEAR_TIE_FP32 = 0.01  # fp32 residual stream
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -23,14 +35,20 @@ def _built():
     ensure_built()
 
 
-def _compare(adt, ref, margins):
-    """Tokens equal up to the end, or up to a near tie of the reference."""
-    for i, (a, r) in enumerate(zip(adt, ref)):
-        if a != r:
-            assert margins[i] < NEAR_TIE, f"token {i}: {a} != {r} with a relative top-2 gap of {margins[i]:.4f}"
-            return i
-    assert len(adt) == len(ref)
-    return len(adt)
+def _check(adt, choice, margins, max_ties, near_tie=NEAR_TIE_BF16):
+    """Every token the tree decoder emitted is the reference's greedy choice
+    at that position, except at near ties (at most max_ties of them)."""
+    assert len(adt) == len(choice)
+    diff = [i for i, (a, r) in enumerate(zip(adt, choice)) if a != r]
+    for i in diff:
+        assert margins[i] < near_tie, f"token {i}: {adt[i]} != {choice[i]}, relative top-2 gap {margins[i]:.4f}"
+    assert len(diff) <= max_ties, f"{len(diff)} near-tie differences"
+    return len(diff)
+
+
+def _reference(shape, weights, prompt, out):
+    """The reference's choice and margin at every position of `out`."""
+    return greedy_decode(shape, weights, prompt, len(out[0]), batch=len(out), return_margins=True, forced=out)
 
 
 def _prompt(vocab, n, seed):
@@ -47,11 +65,10 @@ def test_adt_decode_equals_greedy(batch, graphs):
     dec = Decoder(SMALL, batch=batch, grid=(8, 8), prompt_len=8, seed=7, max_nodes=64, graphs=graphs)
     prompt = _prompt(SMALL.vocab, 8, 1)
     out, stats = dec.generate(prompt)
-    ref, margins = greedy_decode(SMALL, dec.target_w, prompt, 64, batch=batch, return_margins=True, graphs=graphs)
+    choice, margins = _reference(SMALL, dec.target_w, prompt, out)
     for b in range(batch):
         assert len(out[b]) == 64
-        n = _compare(out[b], ref[b], margins[b])
-        assert n >= 16, f"image {b}: only {n} tokens before a near tie"
+        _check(out[b], choice[b], margins[b], max_ties=3)
     assert B.adt_get_device_error() == 0
     assert stats.steps >= 1 and stats.tau >= 1.0
 
@@ -66,9 +83,8 @@ def test_adt_decode_with_a_draft_that_matches_the_target():
                   ctrl_params=dict(d_lo=1, d_hi=6, k_lo=2, k_hi=4))
     prompt = _prompt(shape.vocab, 8, 2)
     out, stats = dec.generate(prompt)
-    ref, margins = greedy_decode(shape, dec.target_w, prompt, 96, return_margins=True)
-    n = _compare(out[0], ref[0], margins[0])
-    assert n >= 24
+    choice, margins = _reference(shape, dec.target_w, prompt, out)
+    _check(out[0], choice[0], margins[0], max_ties=3)
     assert stats.accepted >= stats.steps, "a matching draft should average at least one accepted token per step"
     assert B.adt_get_device_error() == 0
 
@@ -82,7 +98,7 @@ def test_adt_decode_equals_greedy_fp32_stream():
     dec = Decoder(shape, batch=2, grid=(8, 8), prompt_len=12, seed=5, max_nodes=64)
     prompt = _prompt(shape.vocab, 12, 3)
     out, stats = dec.generate(prompt)
-    ref, margins = greedy_decode(shape, dec.target_w, prompt, 64, batch=2, return_margins=True)
+    choice, margins = _reference(shape, dec.target_w, prompt, out)
     for b in range(2):
-        assert _compare(out[b], ref[b], margins[b]) >= 48
+        _check(out[b], choice[b], margins[b], max_ties=1, near_tie=NEAR_TIE_FP32)
     assert B.adt_get_device_error() == 0
