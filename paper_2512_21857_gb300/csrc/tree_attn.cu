@@ -64,6 +64,7 @@ constexpr int kMaxClusterSplits = 8;    // portable cluster size
 constexpr int kMaxSplits = 96;          // workspace merge: weights fit in shared memory
 constexpr int kMaxStages = 4;
 constexpr uint32_t kWaitLimit = 1u << 20;
+constexpr int kTmaRows = 1 << 24;       // node extent of the Q / tree tensor maps (boxes are kept inside the buffers)
 constexpr uint32_t kTmemCols = 512;     // two S tiles of 128 columns, O (<= 128 columns), row sums
 constexpr uint32_t kSCols = 128;
 constexpr uint32_t kOCol = 256;
@@ -258,7 +259,8 @@ __device__ __forceinline__ void chunk_softmax(float (&sa)[32], float (&sb)[32], 
 }
 
 struct Barriers {
-  uint64_t q_full;                 // Q and the tree unit's K/V are in shared memory
+  uint64_t q_full;                 // Q and the tree unit's K/V are in shared memory (softmax warps' copies)
+  uint64_t q_tma;                  // the same, when they come as tensor copies: those copies landed
   uint64_t k_full[kMaxStages];     // a stage's K tile has landed
   uint64_t v_full[kMaxStages];     // a stage's V tile has landed
   uint64_t k_free[kMaxStages];     // the S product of the chunk in that slot finished
@@ -287,10 +289,12 @@ __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, volatil
 
 // kLarge: trees of more than 64 nodes (query tiles, one mask word per tree
 // unit); otherwise one tile and one word, kept in registers.
+
 template <int D, bool kLarge>
 __global__ void __launch_bounds__(kThreads, 1)
     tree_attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
-                        const TcParams p) {
+                        const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kt,
+                        const __grid_constant__ CUtensorMap tm_vt, const TcParams p) {
   using C = Cfg<D>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-byte aligned for the 128-byte swizzle; pointer arithmetic on the
@@ -320,6 +324,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     s_bad = 0;
     s_abort = 0;
     sm100::mbar_init(sm100::smem_addr(&bars.q_full), kSoftmaxWarps);
+    sm100::mbar_init(sm100::smem_addr(&bars.q_tma), 1);
     for (int s = 0; s < NS; ++s) {
       sm100::mbar_init(sm100::smem_addr(&bars.k_full[s]), 1);
       sm100::mbar_init(sm100::smem_addr(&bars.v_full[s]), 1);
@@ -340,8 +345,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     sm100::tmem_alloc(sm100::smem_addr(&tmem_slot), kTmemCols);
     sm100::tmem_relinquish();
   }
-  if ((warp == kKLoadWarp || warp == kVLoadWarp) && lane == 0)
-    sm100::prefetch_tensormap(warp == kVLoadWarp ? &tm_v : &tm_k);
+  if (warp == kKLoadWarp && lane < 4)
+    sm100::prefetch_tensormap(lane == 0 ? &tm_k : lane == 1 ? &tm_q : lane == 2 ? &tm_kt : &tm_vt);
+  if (warp == kVLoadWarp && lane == 0) sm100::prefetch_tensormap(&tm_v);
   sm100::tc_fence_before();
   __syncthreads();
   sm100::tc_fence_after();
@@ -406,8 +412,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int Tc = kLarge ? (qt + 2) / 2 : 1;  // tree chunks of this tile
   const int T = Pc + Tc;
   const int S = p.splits;
-  const int c_begin = static_cast<int>(static_cast<int64_t>(split) * T / S);
-  const int c_end = static_cast<int>(static_cast<int64_t>(split + 1) * T / S);
+  // (32-bit: T < 2^24 chunks and S <= 96 splits; 64-bit division is slow)
+  const int c_begin = split * T / S;
+  const int c_end = (split + 1) * T / S;
   const int nch = c_end - c_begin;
   const int tc0 = max(c_begin, Pc) - Pc;         // first tree chunk of this split
   const int n_tc = max(0, c_end - max(c_begin, Pc));  // its tree chunks, in slots 0 .. n_tc-1
@@ -418,6 +425,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   };
   auto chunk_key0 = [&](int j) -> int { return (c_begin + j - n_tc) * kChunk; };
 
+  // Q (and the one tree unit's K/V) as 64-row tensor copies when the whole
+  // box lies inside the node_offsets[B] rows the caller's buffers hold;
+  // otherwise (the last tree of a batch with fewer than 64 nodes after its
+  // first, or trees of more than 64 nodes) the softmax warps copy the rows
+  // of the tree alone, 16 bytes at a time.
+  const bool q_tma = !kLarge && node0 + kMaxNodes <= total_nodes && total_nodes < kTmaRows;
   uint8_t* sQ = smem + C::kQOff;
   uint8_t* sP = smem + C::kPOff;
   uint8_t* sStage = smem + C::kStageOff;
@@ -427,7 +440,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Q tile: rows row0 .. row0+63 of the tree (rows past it zero-filled);
     // this split's tree chunks (K/V of kv head g, nodes past the tree
     // zero-filled) into stage slots 0 .. n_tc-1; the parent pointers.
-    for (int i = tid; i < kUnit * (D / 8); i += kSoftmaxWarps * 32) {
+    for (int i = tid; !q_tma && i < kUnit * (D / 8); i += kSoftmaxWarps * 32) {
       const int r = i / (D / 8), ch = i % (D / 8);
       const bool valid = r < nq;
       const int row = node0 + row0 + (valid ? r : 0);
@@ -455,13 +468,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     static_assert(C::kOnesBytes == kSoftmaxWarps * 32 * 16, "one 16-byte store per softmax thread");
     reinterpret_cast<uint4*>(smem + C::kOnesOff)[tid] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
   }
-  // Q's copies are requested before the stage loads: a CTA's first stages
-  // are 128 KB, and Q queued behind them would hold back the first S.
-  __syncthreads();
-  // The mbarriers are initialised: tell the cluster (the merge's bulk copies
-  // complete on a peer's barrier; every thread waits on this before one).
-  sm100::cluster_arrive_relaxed();
-
   // Stage loads: chunk j goes to slot j % NS, K tile by warp 4 and V tile by
   // warp 6.  A tree chunk loads nothing (its K/V came with Q) but still
   // completes its slot's phases, so that every slot's phases advance once
@@ -475,19 +481,42 @@ __global__ void __launch_bounds__(kThreads, 1)
       sm100::mbar_arrive(bar);
       return;
     }
-    const int halves = chunk_keys(j) / kUnit;
+    // One 128-key box per column block (a chunk of one unit loads the next
+    // 64 rows too; nothing reads them: its products stop at 64 keys).
     const int key0 = chunk_key0(j);
     uint8_t* dst = sStage + st * C::kStageBytes + (load_v ? C::kStageTile : 0);
     const CUtensorMap* map = load_v ? &tm_v : &tm_k;
-    sm100::mbar_arrive_expect_tx(bar, C::kBlocks * halves * C::kBlock64);
-    for (int blk = 0; blk < C::kBlocks; ++blk) {
-      for (int hf = 0; hf < halves; ++hf)
-        sm100::tma_load_4d(sm100::smem_addr(dst + blk * C::kBlock128 + hf * C::kBlock64), map, blk * 64,
-                           key0 + hf * kUnit, g, b, bar);
-    }
+    sm100::mbar_arrive_expect_tx(bar, C::kBlocks * C::kBlock128);
+    for (int blk = 0; blk < C::kBlocks; ++blk)
+      sm100::tma_load_4d(sm100::smem_addr(dst + blk * C::kBlock128), map, blk * 64, key0, g, b, bar);
   };
   const int first_issue = nch < NS ? nch : NS;
-  if (is_loader) {
+  if (q_tma) {
+    // Q and the tree unit go out first, from the thread that then requests
+    // the first K stages; nothing waits for the softmax warps' set-up.
+    if (warp == kKLoadWarp && lane == 0) {
+      const uint32_t bar = sm100::smem_addr(&bars.q_tma);
+      sm100::mbar_arrive_expect_tx(bar, C::kBlocks * C::kBlock64 * (n_tc ? 3 : 1));
+      for (int blk = 0; blk < C::kBlocks; ++blk)
+        sm100::tma_load_3d(sm100::smem_addr(sQ + blk * C::kBlock64), &tm_q, blk * 64, h, node0, bar);
+      for (int blk = 0; n_tc && blk < C::kBlocks; ++blk) {
+        sm100::tma_load_3d(sm100::smem_addr(sStage + blk * C::kBlock128), &tm_kt, blk * 64, g, node0, bar);
+        sm100::tma_load_3d(sm100::smem_addr(sStage + C::kStageTile + blk * C::kBlock128), &tm_vt, blk * 64, g, node0,
+                           bar);
+      }
+    }
+    if (is_loader) {
+      for (int j = 0; j < first_issue; ++j) issue_tile(j);
+    }
+  }
+  // Q's copies (when the softmax warps make them) are requested before the
+  // stage loads: a CTA's first stages are 128 KB, and Q queued behind them
+  // would hold back the first S.
+  __syncthreads();
+  // The mbarriers are initialised: tell the cluster (the merge's bulk copies
+  // complete on a peer's barrier; every thread waits on this before one).
+  sm100::cluster_arrive_relaxed();
+  if (!q_tma && is_loader) {
     for (int j = 0; j < first_issue; ++j) issue_tile(j);
   }
   if (warp < kSoftmaxWarps) {
@@ -563,6 +592,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = 0; j < first_issue; ++j)
         (void)sm100::mbar_wait_bounded(sm100::smem_addr(load_v ? &bars.v_full[j % NS] : &bars.k_full[j % NS]), 0,
                                        kWaitLimit);
+      if (q_tma && !load_v) (void)sm100::mbar_wait_bounded(sm100::smem_addr(&bars.q_tma), 0, kWaitLimit);
     }
     sm100::tc_fence_before();
     __syncthreads();
@@ -591,12 +621,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = (issued > NS ? issued - NS : 0); j < issued; ++j)
         (void)sm100::mbar_wait_bounded(sm100::smem_addr(load_v ? &bars.v_full[j % NS] : &bars.k_full[j % NS]),
                                        (j / NS) & 1, kWaitLimit);
+      if (q_tma && !load_v) (void)sm100::mbar_wait_bounded(sm100::smem_addr(&bars.q_tma), 0, kWaitLimit);
     }
     __syncwarp();
   } else if (warp == kSMmaWarp) {
     // ------------------------------------------------------------ S = Q K^T
     if (lane == 0) {
-      bool ok = wait_bar(&bars.q_full, 0, &s_abort, p.err, p.wait_limit);
+      bool ok = wait_bar(&bars.q_full, 0, &s_abort, p.err, p.wait_limit) &&
+                (!q_tma || wait_bar(&bars.q_tma, 0, &s_abort, p.err, p.wait_limit));
       const uint32_t q_addr = sm100::smem_addr(sQ);
       for (int j = 0; ok && j < nch; ++j) {
         const int st = j % NS, sb = j & 1;
@@ -650,6 +682,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else {
     // ------------------------------------------------------------ softmax warps 0-3
+    if (q_tma && n_tc && n < kUnit) {
+      // The tree unit came as a 64-row box: V rows past the tree (another
+      // tree's nodes) are zeroed, so that P = 0 there meets finite values.
+      if (__all_sync(adt::kFullMask, wait_bar(&bars.q_tma, 0, &s_abort, p.err, p.wait_limit))) {
+        uint8_t* vt = sStage + C::kStageTile;
+        const int per_row = C::kBlocks * 8;
+        for (int i = tid; i < (kUnit - n) * per_row; i += kSoftmaxWarps * 32) {
+          const int rr = n + i / per_row, rem = i % per_row;
+          *reinterpret_cast<uint4*>(vt + (rem >> 3) * C::kBlock128 + rr * 128 + (rem & 7) * 16) =
+              make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
+    }
     sm100::fence_proxy_async_smem();
     __syncwarp();
     if (lane == 0) sm100::mbar_arrive(sm100::smem_addr(&bars.q_full));
@@ -1088,7 +1133,8 @@ void load_encode() {
 }
 
 // 4-D map of a cache (d, pos, kv head, tree) with the 128-byte swizzle and
-// 64 x 64 boxes; positions at or past max_kv read as zero.
+// boxes of 64 columns x 128 positions; positions at or past max_kv read as
+// zero.
 adt_status make_cache_map(CUtensorMap* map, const void* base, int D, int max_kv, int Hkv, int B, int64_t sh,
                           int64_t sb) {
   std::call_once(g_encode_once, load_encode);
@@ -1098,9 +1144,26 @@ adt_status make_cache_map(CUtensorMap* map, const void* base, int D, int max_kv,
                         static_cast<cuuint64_t>(B)};
   cuuint64_t strides[3] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(sh > 0 ? sh : span * D) * 2,
                            static_cast<cuuint64_t>(sb > 0 ? sb : span * D * Hkv) * 2};
-  cuuint32_t box[4] = {64, kUnit, 1, 1};
+  cuuint32_t box[4] = {64, kChunk, 1, 1};
   cuuint32_t estr[4] = {1, 1, 1, 1};
   CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? ADT_OK : ADT_ERR_INVALID_ARG;
+}
+
+// 3-D map of a node-major tensor [nodes][heads][D] (Q or the tree's K / V)
+// with the 128-byte swizzle and boxes of 64 nodes x 64 columns of one head.
+// The node extent is nominal: the kernel only requests boxes that lie inside
+// the node_offsets[B] rows the caller's buffer holds.
+adt_status make_rows_map(CUtensorMap* map, const void* base, int D, int heads) {
+  std::call_once(g_encode_once, load_encode);
+  if (!g_encode) return ADT_ERR_CUDA;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(heads), static_cast<cuuint64_t>(kTmaRows)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(heads) * D * 2};
+  cuuint32_t box[3] = {64, 1, kUnit};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? ADT_OK : ADT_ERR_INVALID_ARG;
@@ -1150,11 +1213,14 @@ adt_status launch(TcParams prm, const void* k_cache, const void* v_cache, int64_
                                       Cfg<D>::kDynSmem));
     __atomic_fetch_or(&word, bit, __ATOMIC_ACQ_REL);
   }
-  CUtensorMap tm_k, tm_v;
+  CUtensorMap tm_k, tm_v, tm_q, tm_kt, tm_vt;
   adt_status s1 = make_cache_map(&tm_k, k_cache, D, prm.max_kv, prm.Hkv, prm.B, sh, sb);
   if (s1 != ADT_OK) return s1;
   s1 = make_cache_map(&tm_v, v_cache, D, prm.max_kv, prm.Hkv, prm.B, sh, sb);
   if (s1 != ADT_OK) return s1;
+  if ((s1 = make_rows_map(&tm_q, prm.q, D, prm.H)) != ADT_OK) return s1;
+  if ((s1 = make_rows_map(&tm_kt, prm.kt, D, prm.Hkv)) != ADT_OK) return s1;
+  if ((s1 = make_rows_map(&tm_vt, prm.vt, D, prm.Hkv)) != ADT_OK) return s1;
   prm.cluster_merge = prm.splits <= kMaxClusterSplits ? 1 : 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(prm.splits), static_cast<unsigned>(prm.H),
@@ -1173,7 +1239,7 @@ adt_status launch(TcParams prm, const void* k_cache, const void* v_cache, int64_
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = overlap_previous ? 2 : 1;
-  ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, tree_attn_tc_kernel<D, kLarge>, tm_k, tm_v, prm));
+  ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, tree_attn_tc_kernel<D, kLarge>, tm_k, tm_v, tm_q, tm_kt, tm_vt, prm));
   return adt::launch_status();
 }
 
@@ -1394,3 +1460,4 @@ extern "C" adt_status adt_tree_attn_noalloc(const adt_bf16* q, const adt_bf16* k
   prm.tickets = reinterpret_cast<unsigned*>(ws + w.tickets);
   return launch_any(prm, D, k_cache, v_cache, cache_stride_b, cache_stride_h, s, info.device, false);
 }
+
