@@ -115,6 +115,13 @@ const char* adt_status_string(adt_status s);
  * calls on other threads. */
 adt_status adt_testing_set_wait_limit(uint32_t polls);
 
+/* Testing hook, not for production use: out[i] = e^(a[i] - b[i]) (a[i] <= b[i])
+ * as the sampling modes of adt_tree_accept compute it, in double-float
+ * arithmetic (two fp32 words; table-driven reduction), returned as fp64, so
+ * that a test can bound its error against an fp64 exponential.  a, b
+ * [device] fp32 [n]; out [device] fp64 [n]. */
+adt_status adt_testing_exp_diff(const float* a, const float* b, int32_t n, double* out, void* stream);
+
 /* ------------------------------------------------------------------------
  * adt_tree_attn - tree-masked attention for one transformer layer.
  *

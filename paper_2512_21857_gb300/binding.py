@@ -24,7 +24,7 @@ INIT_HORIZONTAL, INIT_VERTICAL, INIT_RANDOM, INIT_TOKENFLOCK = 0, 1, 2, 3
 DEVERR_BAD_TREE, DEVERR_KV_RANGE, DEVERR_BAD_PATH, DEVERR_TIMEOUT, DEVERR_BAD_INDEX = 1, 2, 4, 8, 16
 
 EXPORTED = [
-    "adt_version", "adt_get_device_error", "adt_status_string", "adt_testing_set_wait_limit",
+    "adt_version", "adt_get_device_error", "adt_status_string", "adt_testing_set_wait_limit", "adt_testing_exp_diff",
     "adt_tree_attn_workspace_size", "adt_tree_attn", "adt_tree_attn_noalloc",
     "adt_tree_expand_workspace_size", "adt_tree_expand", "adt_tree_expand_cfg",
     "adt_tree_rerank_workspace_size", "adt_tree_rerank",
@@ -56,6 +56,7 @@ _SIGS = {
     "adt_get_device_error": ([_P, ctypes.POINTER(ctypes.c_uint32)], _I32),
     "adt_status_string": ([_I32], ctypes.c_char_p),
     "adt_testing_set_wait_limit": ([ctypes.c_uint32], _I32),
+    "adt_testing_exp_diff": ([_P, _P, _I32, _P, _P], _I32),
     "adt_tree_attn_workspace_size": ([_I32] * 5, _SZ),
     "adt_tree_attn": ([_P, _P, _P, _P, _I64, _I64, _P, _P, _P, _P, _I32, _I32, _I32, _I32, _I32, _I32, _F32,
                        _P, _P, _P, _SZ, _P], _I32),
@@ -151,6 +152,12 @@ def adt_get_device_error(stream=None) -> int:
 def adt_testing_set_wait_limit(polls: int) -> None:
     """Testing hook: polls before adt_tree_attn's pipeline waits give up (0 = default)."""
     _check(lib().adt_testing_set_wait_limit(int(polls)), "adt_testing_set_wait_limit")
+
+
+def adt_testing_exp_diff(a, b, out, stream=None) -> None:
+    """Testing hook: out = e^(a - b) in the acceptance walk's double-float arithmetic."""
+    _check(lib().adt_testing_exp_diff(_ptr(a), _ptr(b), int(a.numel()), _ptr(out), _stream(stream)),
+           "adt_testing_exp_diff")
 
 
 def adt_tree_attn_workspace_size(B, H, D, max_nodes, max_kv) -> int:

@@ -15,6 +15,7 @@
 #include <cooperative_groups.h>
 
 #include "adt_common.cuh"
+#include "dfloat.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -65,9 +66,15 @@ struct Shared {
   int kids[kMaxNodes];
   int path[kMaxNodes];
   int rejected[kMaxNodes];
-  double dred[32];
   float fred[32];
   int ired[32];
+  float2 exptab[64];  // 2^(j/64) as double-floats (the double-float exponential's table)
+  float2 dfred[32];   // double-float block reductions
+  // Scalars thread 0 derives from the cluster's published values (in fp64,
+  // once per CTA: FP64 runs at a small fraction of the FP32 rate, so every
+  // thread repeating them would cost microseconds) and hands to the block.
+  float2 bf[4];
+  int bi[4];
   int nkids;
   int bad;
   int found;
@@ -90,6 +97,68 @@ struct Walker {
 __device__ __forceinline__ bool better(float v, int i, float bv, int bi) {
   return v > bv || (v == bv && i < bi);
 }
+
+// The sampling modes' slices of p and q.  Slice<true>: double-float
+// entries (hi, lo), exponentials and every update in double-float, so the
+// decisions the walk takes from them (u q(x) < p(x), the inverse-CDF draw)
+// agree with fp64 arithmetic to about 1e-11 relative; used where the slices
+// fit in shared memory.  Slice<false>: fp32 entries and fp32 exponentials
+// (relative error about 1e-7), for larger vocabularies.
+template <bool kDF>
+struct Slice;
+
+template <>
+struct Slice<false> {
+  using E = float;
+  static __device__ __forceinline__ E logit(float x) { return x; }
+  static __device__ __forceinline__ float value_hi(E v) { return v; }
+  static __device__ __forceinline__ E exp_diff(float x, float M, const float2*) { return expf(x - M); }
+  static __device__ __forceinline__ double d(E v) { return v; }
+  static __device__ __forceinline__ bool pos(E v) { return v > 0.f; }
+  static __device__ __forceinline__ E zero() { return 0.f; }
+  static __device__ __forceinline__ dfl::df as_df(E v) { return dfl::df{v, 0.f}; }
+  using F = float;  // a scale factor, converted once per pass
+  static __device__ __forceinline__ F factor(float2 s) { return s.x; }
+  static __device__ __forceinline__ E scale(E v, F f) { return v * f; }
+  static __device__ __forceinline__ E resid(E p, E q) { return fmaxf(p - q, 0.f); }
+  struct Acc {
+    float a = 0.f;
+    __device__ __forceinline__ void add(E v) { a += v; }
+    __device__ __forceinline__ double value() const { return a; }
+    __device__ __forceinline__ dfl::df value_df() const { return dfl::df{a, 0.f}; }
+  };
+};
+
+template <>
+struct Slice<true> {
+  using E = float2;
+  static __device__ __forceinline__ E logit(float x) { return make_float2(x, 0.f); }
+  static __device__ __forceinline__ float value_hi(E v) { return v.x; }
+  static __device__ __forceinline__ E exp_diff(float x, float M, const float2* tab) {
+    const dfl::df e = dfl::df_exp_diff(x, M, tab);
+    return make_float2(e.hi, e.lo);
+  }
+  static __device__ __forceinline__ double d(E v) { return static_cast<double>(v.x) + static_cast<double>(v.y); }
+  static __device__ __forceinline__ bool pos(E v) { return v.x > 0.f; }
+  static __device__ __forceinline__ E zero() { return make_float2(0.f, 0.f); }
+  static __device__ __forceinline__ dfl::df as_df(E v) { return dfl::df{v.x, v.y}; }
+  using F = dfl::df;
+  static __device__ __forceinline__ F factor(float2 s) { return dfl::df{s.x, s.y}; }
+  static __device__ __forceinline__ E scale(E v, F f) {
+    const dfl::df r = dfl::df_mul(dfl::df{v.x, v.y}, f);
+    return make_float2(r.hi, r.lo);
+  }
+  static __device__ __forceinline__ E resid(E p, E q) {
+    const dfl::df r = dfl::df_max0(dfl::df_add(dfl::df{p.x, p.y}, dfl::df{-q.x, -q.y}));
+    return make_float2(r.hi, r.lo);
+  }
+  struct Acc {
+    dfl::Acc a;
+    __device__ __forceinline__ void add(E v) { a.add(dfl::df{v.x, v.y}); }
+    __device__ __forceinline__ double value() const { return a.value(); }
+    __device__ __forceinline__ dfl::df value_df() const { return a.value_df(); }
+  };
+};
 
 // Block argmax over (value desc, index asc); all threads get the result.
 __device__ void block_argmax(float& v, int& idx, Shared* sh) {
@@ -123,8 +192,9 @@ __device__ void block_argmax(float& v, int& idx, Shared* sh) {
 // Loads this CTA's slice of a logit row (under guidance u + s (c - u) with
 // the unconditional row row_u; then divided by T) into buf; entries past V
 // are -inf.
-__device__ void load_slice(const float* row, const float* row_u, int lo, int cnt, int Vs, float* buf,
-                           const AcceptParams& p) {
+template <bool kDF>
+__device__ void load_slice(const float* row, const float* row_u, int lo, int cnt, int Vs,
+                           typename Slice<kDF>::E* buf, const AcceptParams& p) {
   for (int i = threadIdx.x * 4; i < Vs; i += kThreads * 4) {
     float x[4];
     if (i + 3 < cnt) {
@@ -147,56 +217,75 @@ __device__ void load_slice(const float* row, const float* row_u, int lo, int cnt
     for (int e = 0; e < 4; ++e) {
       float y = x[e];
       if (p.use_T && i + e < cnt) y = __fdiv_rn(y, p.T);
-      buf[i + e] = y;
+      buf[i + e] = Slice<kDF>::logit(y);
     }
   }
 }
 
-// exp(x - M) in place over the slice; returns the block's sum (fp64 from
-// per-thread fp32 partials).
-__device__ double exp_in_place(float* buf, int Vs, float M, Shared* sh) {
-  float acc = 0.f;
-  for (int i = threadIdx.x; i < Vs; i += kThreads) {
-    const float e = expf(buf[i] - M);
-    buf[i] = e;
-    acc += e;
-  }
-  return adt::block_sum<kThreads, double>(static_cast<double>(acc), sh->dred);
+// Sum over the block in double-float (fp32 operations only); every thread
+// gets the result.
+__device__ dfl::df block_sum_df(dfl::df v, Shared* sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int o = 16; o > 0; o >>= 1)
+    v = dfl::df_add(v, dfl::df{__shfl_xor_sync(adt::kFullMask, v.hi, o), __shfl_xor_sync(adt::kFullMask, v.lo, o)});
+  __syncthreads();
+  if (lane == 0) sh->dfred[warp] = make_float2(v.hi, v.lo);
+  __syncthreads();
+  dfl::df r = lane < kThreads / 32 ? dfl::df{sh->dfred[lane].x, sh->dfred[lane].y} : dfl::df{0.f, 0.f};
+  for (int o = 16; o > 0; o >>= 1)
+    r = dfl::df_add(r, dfl::df{__shfl_xor_sync(adt::kFullMask, r.hi, o), __shfl_xor_sync(adt::kFullMask, r.lo, o)});
+  return r;
 }
 
-__device__ float slice_max(const float* buf, int Vs, Shared* sh) {
+// exp(x - M) in place over the slice (the logits M is the row maximum of);
+// returns the block's sum.
+template <bool kDF>
+__device__ dfl::df exp_in_place(typename Slice<kDF>::E* buf, int Vs, float M, Shared* sh) {
+  typename Slice<kDF>::Acc acc;
+  for (int i = threadIdx.x; i < Vs; i += kThreads) {
+    const typename Slice<kDF>::E e = Slice<kDF>::exp_diff(Slice<kDF>::value_hi(buf[i]), M, sh->exptab);
+    buf[i] = e;
+    acc.add(e);
+  }
+  return block_sum_df(acc.value_df(), sh);
+}
+
+template <bool kDF>
+__device__ float slice_max(const typename Slice<kDF>::E* buf, int Vs, Shared* sh) {
   float m = -INFINITY;
-  for (int i = threadIdx.x; i < Vs; i += kThreads) m = fmaxf(m, buf[i]);
+  for (int i = threadIdx.x; i < Vs; i += kThreads) m = fmaxf(m, Slice<kDF>::value_hi(buf[i]));
   return adt::block_max<kThreads>(m, sh->fred);
 }
 
 // Inverse-CDF draw over the (unnormalised, non-negative) distribution held
 // in the cluster's slices: smallest t with sum_{j<=t} w_j > u * sum_j w_j.
 // Returns the token id on every CTA.
-__device__ int cluster_sample(Walker& w, const float* buf, int lo, int cnt, double u, Shared* sh) {
+template <bool kDF>
+__device__ int cluster_sample(Walker& w, const typename Slice<kDF>::E* buf, int lo, int cnt, double u, Shared* sh) {
   // 1. per-CTA slice totals (each thread owns a contiguous run), published.
   const int per = (cnt + kThreads - 1) / kThreads;
   const int b0 = min(cnt, static_cast<int>(threadIdx.x) * per), b1 = min(cnt, b0 + per);
-  double run = 0.0;
+  typename Slice<kDF>::Acc racc;
   int last_pos = -1;
   for (int i = b0; i < b1; ++i) {
-    run += buf[i];
-    if (buf[i] > 0.f) last_pos = i;
+    racc.add(buf[i]);
+    if (Slice<kDF>::pos(buf[i])) last_pos = i;
   }
-  const double tot = adt::block_sum<kThreads, double>(run, sh->dred);
-  if (threadIdx.x == 0) w.publish_slot()->d[0] = tot;
+  const dfl::df run = racc.value_df();
+  const dfl::df tot = block_sum_df(run, sh);
+  if (threadIdx.x == 0) w.publish_slot()->d[0] = dfl::to_double(tot);
   w.exchange();
-  double grand = 0.0, base = 0.0;
-  for (int c = 0; c < w.csize; ++c) {
-    const double t = w.peer(c)->d[0];
-    if (c < w.rank) base += t;
-    grand += t;
-  }
-  const double target = u * grand;
-  // Owner: first CTA whose cumulative total passes the target; else the last
-  // CTA with mass.
-  int owner = -1, last_nz = -1;
-  {
+  if (threadIdx.x == 0) {
+    double grand = 0.0, base = 0.0;
+    for (int c = 0; c < w.csize; ++c) {
+      const double t = w.peer(c)->d[0];
+      if (c < w.rank) base += t;
+      grand += t;
+    }
+    const double target = u * grand;
+    // Owner: first CTA whose cumulative total passes the target; else the
+    // last CTA with mass.
+    int owner = -1, last_nz = -1;
     double acc = 0.0;
     for (int c = 0; c < w.csize; ++c) {
       const double t = w.peer(c)->d[0];
@@ -204,33 +293,40 @@ __device__ int cluster_sample(Walker& w, const float* buf, int lo, int cnt, doub
       if (t > 0.0) last_nz = c;
       acc += t;
     }
-    if (owner < 0) owner = last_nz < 0 ? 0 : last_nz;
+    sh->bi[0] = owner < 0 ? (last_nz < 0 ? 0 : last_nz) : owner;
+    const dfl::df bdf = dfl::from_double(base), tdf = dfl::from_double(-target);
+    sh->bf[0] = make_float2(bdf.hi, bdf.lo);
+    sh->bf[1] = make_float2(tdf.hi, tdf.lo);
   }
+  __syncthreads();
+  const int owner = sh->bi[0];
+  const dfl::df base = dfl::df{sh->bf[0].x, sh->bf[0].y}, ntgt = dfl::df{sh->bf[1].x, sh->bf[1].y};
   w.flip();
   int result_local = -1;
   if (w.rank == owner) {
-    // exclusive scan of the per-thread runs
+    // exclusive scan of the per-thread runs, in double-float
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    double incl = run;
+    dfl::df incl = run;
     for (int o = 1; o < 32; o <<= 1) {
-      const double y = __shfl_up_sync(adt::kFullMask, incl, o);
-      if (lane >= o) incl += y;
+      const dfl::df y{__shfl_up_sync(adt::kFullMask, incl.hi, o), __shfl_up_sync(adt::kFullMask, incl.lo, o)};
+      if (lane >= o) incl = dfl::df_add(incl, y);
     }
     __syncthreads();
-    if (lane == 31) sh->dred[warp] = incl;
+    if (lane == 31) sh->dfred[warp] = make_float2(incl.hi, incl.lo);
     if (threadIdx.x == 0) {
       sh->found = 0x7fffffff;
       sh->last_pos = -1;
     }
     __syncthreads();
-    double wbase = 0.0;
-    for (int j = 0; j < warp; ++j) wbase += sh->dred[j];
-    double acc = base + wbase + incl - run;
+    dfl::df acc = base;
+    for (int j = 0; j < warp; ++j) acc = dfl::df_add(acc, dfl::df{sh->dfred[j].x, sh->dfred[j].y});
+    // The running CDF in double-float, compared with the target through the
+    // sign of their difference.
+    acc = dfl::df_add(acc, dfl::df_add(incl, dfl::df_neg(run)));
     if (last_pos >= 0) atomicMax(&sh->last_pos, last_pos);
     for (int i = b0; i < b1; ++i) {
-      const double wv = buf[i];
-      acc += wv;
-      if (acc > target && wv > 0.0) {
+      acc = dfl::df_add(acc, Slice<kDF>::as_df(buf[i]));
+      if (Slice<kDF>::pos(buf[i]) && dfl::df_add(acc, ntgt).hi > 0.f) {
         atomicMin(&sh->found, i);
         break;
       }
@@ -247,16 +343,20 @@ __device__ int cluster_sample(Walker& w, const float* buf, int lo, int cnt, doub
   return res;
 }
 
+template <bool kDF>
 __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) {
+  using SL = Slice<kDF>;
+  using E = typename SL::E;
   extern __shared__ __align__(16) float dyn[];
   __shared__ Shared sh;
+  if (kDF) dfl::exp_table_to_smem(sh.exptab);  // read after the __syncthreads below
   adt::pdl_wait_then_release();
   cg::cluster_group cl = cg::this_cluster();
   Walker w{cl, &sh, static_cast<int>(cl.block_rank()), static_cast<int>(cl.num_blocks()), 0};
   const int b = blockIdx.x / w.csize;
   const int tid = threadIdx.x;
-  float* pbuf = dyn;
-  float* qbuf = dyn + p.Vs;
+  E* pbuf = reinterpret_cast<E*>(dyn);
+  E* qbuf = pbuf + p.Vs;
   const int lo = w.rank * p.Vs;
   const int cnt = max(0, min(p.Vs, p.V - lo));
 
@@ -370,12 +470,12 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
       nk = 0;
     }
     const bool need_q = spec && nk > 0;
-    load_slice(trow, trow_u, lo, cnt, p.Vs, pbuf, p);
+    load_slice<kDF>(trow, trow_u, lo, cnt, p.Vs, pbuf, p);
     if (need_q)
-      load_slice(p.draft + dr * p.ldd, p.draft_u ? p.draft_u + dr * p.ldd : nullptr, lo, cnt, p.Vs, qbuf, p);
+      load_slice<kDF>(p.draft + dr * p.ldd, p.draft_u ? p.draft_u + dr * p.ldd : nullptr, lo, cnt, p.Vs, qbuf, p);
     __syncthreads();
-    const float mp = slice_max(pbuf, p.Vs, &sh);
-    const float mq = need_q ? slice_max(qbuf, p.Vs, &sh) : 0.f;
+    const float mp = slice_max<kDF>(pbuf, p.Vs, &sh);
+    const float mq = need_q ? slice_max<kDF>(qbuf, p.Vs, &sh) : 0.f;
     if (tid == 0) {
       w.publish_slot()->f[0] = mp;
       w.publish_slot()->f[1] = mq;
@@ -387,33 +487,43 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
       Mq = fmaxf(Mq, w.peer(c)->f[1]);
     }
     w.flip();
-    const double sp_loc = exp_in_place(pbuf, p.Vs, Mp, &sh);
-    const double sq_loc = need_q ? exp_in_place(qbuf, p.Vs, Mq, &sh) : 0.0;
+    const dfl::df sp_loc = exp_in_place<kDF>(pbuf, p.Vs, Mp, &sh);
+    const dfl::df sq_loc = need_q ? exp_in_place<kDF>(qbuf, p.Vs, Mq, &sh) : dfl::df{0.f, 0.f};
     if (tid == 0) {
-      w.publish_slot()->d[0] = sp_loc;
-      w.publish_slot()->d[1] = sq_loc;
+      w.publish_slot()->d[0] = dfl::to_double(sp_loc);
+      w.publish_slot()->d[1] = dfl::to_double(sq_loc);
     }
     w.exchange();
+    // The row totals, formed once (thread 0 keeps them for the decisions) and
+    // handed to the block as double-float reciprocals.
     double Sp = 0.0, Sq = 0.0;
-    for (int c = 0; c < w.csize; ++c) {
-      Sp += w.peer(c)->d[0];
-      Sq += w.peer(c)->d[1];
+    if (tid == 0) {
+      for (int c = 0; c < w.csize; ++c) {
+        Sp += w.peer(c)->d[0];
+        Sq += w.peer(c)->d[1];
+      }
+      const dfl::df ip = dfl::from_double(1.0 / Sp), iq = dfl::from_double(Sq > 0.0 ? 1.0 / Sq : 0.0);
+      sh.bf[0] = make_float2(ip.hi, ip.lo);
+      sh.bf[1] = make_float2(iq.hi, iq.lo);
     }
+    __syncthreads();
     w.flip();
     if (spec && need_q) {
-      // normalise both slices (fp32)
-      const float ip = static_cast<float>(1.0 / Sp), iq = static_cast<float>(1.0 / Sq);
+      // normalise both slices
+      const typename SL::F ip = SL::factor(sh.bf[0]), iq = SL::factor(sh.bf[1]);
       for (int i = tid; i < p.Vs; i += kThreads) {
-        pbuf[i] *= ip;
-        qbuf[i] *= iq;
+        pbuf[i] = SL::scale(pbuf[i], ip);
+        qbuf[i] = SL::scale(qbuf[i], iq);
       }
       w.exchange();  // slices final before any peer reads them
       w.flip();
     }
 
+    // The children in ascending index.  Thread 0 reads p(x), q(x) from the
+    // owning CTA, takes the decision in fp64 and hands it to the block.
     int nxt = -1;
-    double e_rej = 0.0;  // SPEC_DET: rejected unnormalised mass
-    int nrej = 0;
+    double e_rej = 0.0;  // SPEC_DET, thread 0: rejected unnormalised mass
+    int nrej = 0;        // SPEC_DET: rejected tokens (in sh.rejected)
     for (int j = 0; j < nk; ++j) {
       const int c = sh.kids[j];
       const int x = sh.tok[c];
@@ -422,55 +532,69 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
         continue;
       }
       const int owner = x / p.Vs, off = x - owner * p.Vs;
-      const double u = static_cast<double>(p.ua[node0 + c]);
-      bool acc;
-      if (!spec) {
-        bool dup = false;
-        for (int r = 0; r < nrej; ++r) dup |= sh.rejected[r] == x;
-        const double ex = dup ? 0.0 : static_cast<double>(*cl.map_shared_rank(pbuf + off, owner));
-        const double denom = Sp - e_rej;
-        const double px = denom > 0.0 ? ex / denom : 0.0;
-        acc = u < px;
-        if (!acc && !dup) {
-          e_rej += ex;
-          if (tid == 0) sh.rejected[nrej] = x;
-          ++nrej;
-          __syncthreads();
+      if (tid == 0) {
+        const double u = static_cast<double>(p.ua[node0 + c]);
+        if (!spec) {
+          bool dup = false;
+          for (int r = 0; r < nrej; ++r) dup |= sh.rejected[r] == x;
+          const double ex = dup ? 0.0 : SL::d(*cl.map_shared_rank(pbuf + off, owner));
+          const double denom = Sp - e_rej;
+          const double px = denom > 0.0 ? ex / denom : 0.0;
+          const bool a = u < px;
+          sh.bi[1] = a;
+          sh.bi[2] = !a && !dup;  // a new rejected token
+          if (!a && !dup) {
+            e_rej += ex;
+            sh.rejected[nrej] = x;
+          }
+        } else {
+          const double px = SL::d(*cl.map_shared_rank(pbuf + off, owner));
+          const double qx = SL::d(*cl.map_shared_rank(qbuf + off, owner));
+          sh.bi[1] = u * qx < px;
+          sh.bi[2] = 0;
         }
-      } else {
-        const double px = *cl.map_shared_rank(pbuf + off, owner);
-        const double qx = *cl.map_shared_rank(qbuf + off, owner);
-        acc = u * qx < px;
-        if (!acc) {
-          // residual: p <- max(0, p - q)/Z (kept if Z = 0); q(x) <- 0, q <- q/sum
-          float zl = 0.f, ql = 0.f;
-          for (int i = tid; i < p.Vs; i += kThreads) {
-            zl += fmaxf(pbuf[i] - qbuf[i], 0.f);
-            ql += (lo + i == x) ? 0.f : qbuf[i];
-          }
-          const double zb = adt::block_sum<kThreads, double>(static_cast<double>(zl), sh.dred);
-          const double qb = adt::block_sum<kThreads, double>(static_cast<double>(ql), sh.dred);
-          if (tid == 0) {
-            w.publish_slot()->d[0] = zb;
-            w.publish_slot()->d[1] = qb;
-          }
-          w.exchange();  // also: every peer has finished reading px, qx
+      }
+      __syncthreads();
+      const bool acc = sh.bi[1] != 0;
+      nrej += sh.bi[2];
+      __syncthreads();  // sh.bi is rewritten for the next child
+      if (!acc && spec) {
+        // residual: p <- max(0, p - q)/Z (kept if Z = 0); q(x) <- 0, q <- q/sum
+        typename SL::Acc zl, ql;
+        for (int i = tid; i < p.Vs; i += kThreads) {
+          zl.add(SL::resid(pbuf[i], qbuf[i]));
+          if (lo + i != x) ql.add(qbuf[i]);
+        }
+        const dfl::df zb = block_sum_df(zl.value_df(), &sh);
+        const dfl::df qb = block_sum_df(ql.value_df(), &sh);
+        if (tid == 0) {
+          w.publish_slot()->d[0] = dfl::to_double(zb);
+          w.publish_slot()->d[1] = dfl::to_double(qb);
+        }
+        w.exchange();  // also: every peer has finished reading px, qx
+        if (tid == 0) {
           double Z = 0.0, Qs = 0.0;
           for (int cc = 0; cc < w.csize; ++cc) {
             Z += w.peer(cc)->d[0];
             Qs += w.peer(cc)->d[1];
           }
-          w.flip();
-          const float iz = Z > 0.0 ? static_cast<float>(1.0 / Z) : 0.f;
-          const float iqs = Qs > 0.0 ? static_cast<float>(1.0 / Qs) : 0.f;
-          for (int i = tid; i < p.Vs; i += kThreads) {
-            const float pi = pbuf[i], qi = qbuf[i];
-            if (Z > 0.0) pbuf[i] = fmaxf(pi - qi, 0.f) * iz;
-            qbuf[i] = (lo + i == x) ? 0.f : qi * iqs;
-          }
-          w.exchange();  // updated slices visible before the next read
-          w.flip();
+          const dfl::df iz = dfl::from_double(Z > 0.0 ? 1.0 / Z : 0.0);
+          const dfl::df iqs = dfl::from_double(Qs > 0.0 ? 1.0 / Qs : 0.0);
+          sh.bf[0] = make_float2(iz.hi, iz.lo);
+          sh.bf[1] = make_float2(iqs.hi, iqs.lo);
+          sh.bi[0] = Z > 0.0;
         }
+        __syncthreads();
+        w.flip();
+        const typename SL::F iz = SL::factor(sh.bf[0]), iqs = SL::factor(sh.bf[1]);
+        const bool zpos = sh.bi[0] != 0;
+        for (int i = tid; i < p.Vs; i += kThreads) {
+          const E pi = pbuf[i], qi = qbuf[i];
+          if (zpos) pbuf[i] = SL::scale(SL::resid(pi, qi), iz);
+          qbuf[i] = (lo + i == x) ? SL::zero() : SL::scale(qi, iqs);
+        }
+        w.exchange();  // updated slices visible before the next read
+        w.flip();
       }
       if (acc) {
         nxt = c;
@@ -488,11 +612,11 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
       __syncthreads();
       for (int r = 0; r < nrej; ++r) {
         const int x = sh.rejected[r];
-        if (x >= lo && x < lo + cnt && tid == 0) pbuf[x - lo] = 0.f;
+        if (x >= lo && x < lo + cnt && tid == 0) pbuf[x - lo] = SL::zero();
       }
     }
     __syncthreads();
-    bonus = cluster_sample(w, pbuf, lo, cnt, static_cast<double>(p.us[gv]), &sh);
+    bonus = cluster_sample<kDF>(w, pbuf, lo, cnt, static_cast<double>(p.us[gv]), &sh);
     break;
   }
 
@@ -507,7 +631,14 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
   cl.sync();  // no CTA leaves while a peer may still read its shared memory
 }
 
-int cluster_size_for(int V) { return V <= 131072 ? 8 : 16; }
+// 8 CTAs up to 131072 entries for the greedy walk (it keeps no slices);
+// the sampling modes keep slices in shared memory and take 16 CTAs past
+// 65536 entries, so that double-float slices fit up to about 200000 (SPEC)
+// and 262144 (SPEC_DET) entries.
+int cluster_size_for(int V, adt_accept_mode mode) {
+  if (mode == ADT_ACCEPT_GREEDY) return V <= 131072 ? 8 : 16;
+  return V <= 65536 ? 8 : 16;
+}
 
 int slice_for(int V, int cs) {
   int vs = (V + cs - 1) / cs;
@@ -545,21 +676,25 @@ static adt_status accept_impl(const float* target_logits, const float* target_u,
   adt::DeviceInfo info;
   adt_status st = adt::device_info(&info);
   if (st != ADT_OK) return st;
-  const int cs = cluster_size_for(V);
+  const int cs = cluster_size_for(V, mode);
   const int vs = slice_for(V, cs);
-  const size_t smem = static_cast<size_t>(vs) * sizeof(float) * (mode == ADT_ACCEPT_SPEC ? 2 : 1);
+  const int nbuf = mode == ADT_ACCEPT_SPEC ? 2 : 1;
+  // Double-float slices where they fit, fp32 slices otherwise.
+  const size_t smem_df = static_cast<size_t>(vs) * sizeof(float2) * nbuf;
+  const bool use_df = mode != ADT_ACCEPT_GREEDY && smem_df + sizeof(Shared) <= static_cast<size_t>(info.max_smem_optin);
+  const size_t smem = mode == ADT_ACCEPT_GREEDY ? 0 : use_df ? smem_df : static_cast<size_t>(vs) * sizeof(float) * nbuf;
   if (smem + sizeof(Shared) > static_cast<size_t>(info.max_smem_optin)) return ADT_ERR_UNSUPPORTED;
-  static int configured_smem[64];  // largest dynamic smem already allowed, per device
-  static int configured_np[64];
+  static int configured_smem[64][2];  // largest dynamic smem already allowed, per device and instantiation
+  static int configured_np[64][2];
   const int dev = info.device & 63;
-  if (configured_smem[dev] < static_cast<int>(smem)) {
-    ADT_CUDA_TRY(cudaFuncSetAttribute(accept_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      static_cast<int>(smem)));
-    configured_smem[dev] = static_cast<int>(smem);
+  auto kern = use_df ? accept_kernel<true> : accept_kernel<false>;
+  if (configured_smem[dev][use_df] < static_cast<int>(smem)) {
+    ADT_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)));
+    configured_smem[dev][use_df] = static_cast<int>(smem);
   }
-  if (cs > 8 && !configured_np[dev]) {
-    ADT_CUDA_TRY(cudaFuncSetAttribute(accept_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1));
-    configured_np[dev] = 1;
+  if (cs > 8 && !configured_np[dev][use_df]) {
+    ADT_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1));
+    configured_np[dev][use_df] = 1;
   }
   AcceptParams p;
   p.target = target_logits;
@@ -601,11 +736,31 @@ static adt_status accept_impl(const float* target_logits, const float* target_u,
   attr[1] = adt::pdl_attribute();
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, accept_kernel, p));
+  ADT_CUDA_TRY(cudaLaunchKernelEx(&cfg, kern, p));
   return adt::launch_status();
 }
 
+namespace {
+
+__global__ void exp_diff_probe_kernel(const float* a, const float* b, int n, double* out) {
+  __shared__ float2 tab[64];
+  dfl::exp_table_to_smem(tab);
+  __syncthreads();
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
+    out[i] = dfl::to_double(dfl::df_exp_diff(a[i], b[i], tab));
+}
+
+}  // namespace
+
 extern "C" {
+
+adt_status adt_testing_exp_diff(const float* a, const float* b, int32_t n, double* out, void* stream) {
+  ADT_REQUIRE(a && b && out && n >= 0);
+  if (n == 0) return ADT_OK;
+  exp_diff_probe_kernel<<<(n + 255) / 256 < 1024 ? (n + 255) / 256 : 1024, 256, 0, adt::as_stream(stream)>>>(a, b, n,
+                                                                                                         out);
+  return adt::launch_status();
+}
 
 size_t adt_tree_accept_workspace_size(int32_t B, int32_t V) {
   (void)B;
