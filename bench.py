@@ -54,8 +54,8 @@ WORKLOADS = {
 # ncu capture; valid only for the kernel source with this SHA-256 prefix.
 HOST_MARKER = b"// ---------------------------------------------------------------- host side"
 NCU_TRAFFIC = {
-    # dram__bytes_read.sum + dram__bytes_write.sum = 41,495,296 + 0
-    "a7de4b21d9a91d7e": 41495296,
+    # dram__bytes_read.sum + dram__bytes_write.sum = 41,495,040 + 0
+    "084b868da7bc55d9": 41495040,
 }
 
 
@@ -147,6 +147,65 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(use), "samples_in_timed_region": len(inside)}
 
 
+class NvmlSampler:
+    """SM clock and clock-event reasons read through NVML (ctypes on the
+    driver's libnvidia-ml) every ~1 ms in a thread, so that a timed region of
+    a few milliseconds still holds samples.  Reads only."""
+    REASONS = {0x8: "hw_slowdown", 0x40: "hw_thermal_slowdown", 0x20: "sw_thermal_slowdown", 0x4: "sw_power_cap"}
+
+    def __init__(self, device_index):
+        import ctypes
+        import threading
+        self.ok = False
+        self.samples = []
+        self._stop = threading.Event()
+        try:
+            self.lib = ctypes.CDLL("libnvidia-ml.so.1")
+            if self.lib.nvmlInit_v2() != 0:
+                return
+            self.h = ctypes.c_void_p()
+            if self.lib.nvmlDeviceGetHandleByIndex_v2(ctypes.c_uint(device_index), ctypes.byref(self.h)) != 0:
+                return
+            self.max_mhz = ctypes.c_uint(0)
+            self.lib.nvmlDeviceGetMaxClockInfo(self.h, 1, ctypes.byref(self.max_mhz))  # NVML_CLOCK_SM
+            self.ok = True
+        except OSError:
+            return
+        self.thread = threading.Thread(target=self._run, daemon=True)
+
+    def _run(self):
+        import ctypes
+        mhz = ctypes.c_uint(0)
+        reasons = ctypes.c_ulonglong(0)
+        get_reasons = getattr(self.lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            self.lib.nvmlDeviceGetCurrentClocksThrottleReasons
+        while not self._stop.is_set():
+            if self.lib.nvmlDeviceGetClockInfo(self.h, 1, ctypes.byref(mhz)) == 0 and \
+                    get_reasons(self.h, ctypes.byref(reasons)) == 0:
+                self.samples.append((time.time(), mhz.value, reasons.value))
+            time.sleep(0.001)
+
+    def start(self):
+        if self.ok:
+            self.thread.start()
+
+    def stop(self, t0, t1):
+        if not self.ok:
+            return None
+        self._stop.set()
+        self.thread.join(timeout=2)
+        inside = [r for r in self.samples if t0 <= r[0] <= t1]
+        use = inside or self.samples
+        if not use:
+            return None
+        bits = 0
+        for r in use:
+            bits |= r[2]
+        return {"sm_mhz": statistics.median(r[1] for r in use), "sm_max_mhz": self.max_mhz.value,
+                "reasons": sorted(n for m, n in self.REASONS.items() if bits & m), "samples": len(use),
+                "samples_in_timed_region": len(inside), "source": "nvml, 1 ms"}
+
+
 # ------------------------------------------------------------------ GPU arm
 
 def fill_inputs_on_device(step, seed):
@@ -217,6 +276,8 @@ def run_gpu(args, wl, rank, world):
     ea0, ea1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     sampler = ClockSampler(local)
     sampler.start()
+    nvml = NvmlSampler(local)
+    nvml.start()
     time.sleep(0.4)
     if world > 1:
         torch.distributed.barrier()
@@ -239,6 +300,10 @@ def run_gpu(args, wl, rank, world):
     if world > 1:
         torch.distributed.barrier()
     clocks = sampler.stop(t0, t1)
+    fine = nvml.stop(t0, t1)
+    if fine is not None:
+        fine["nvidia_smi"] = clocks
+        clocks = fine
     step_ms = ev0.elapsed_time(ev1) / K
     per_step = sorted(step_ev[i].elapsed_time(step_ev[i + 1]) for i in range(K))
     pct = {f"p{q}": per_step[min(K - 1, int(round(q / 100 * (K - 1))))] for q in (10, 50, 90)}
@@ -498,52 +563,55 @@ def cpu_sample_main(args):
 
 # ------------------------------------------------------------------ main
 
-def run_decode(args):
+def decode_measure(batch, grid, fp32=False, graphs=True):
     """The end-to-end synthetic decode loop (random-init 7B-shape target and
     a one-layer EAGLE-style draft head, ADT-Tree trees every step) over a
-    square image-token grid, timed as a whole, next to vanilla greedy
-    decoding of the same tokens with the same target.  One JSON line."""
+    grid x grid image-token grid, timed as a whole, next to vanilla greedy
+    decoding of the same target in plain torch (no library call; bf16
+    scaled_dot_product_attention), teacher-forced with the tree decoder's
+    tokens so that every emitted token is compared with the target's greedy
+    choice.  Returns a dict of the measurements."""
     import torch
     from paper_2512_21857_gb300 import binding as B
     from paper_2512_21857_gb300 import build
     from paper_2512_21857_gb300.decode import Decoder, ModelShape, greedy_decode
     build.build()
     B.lib()
-    shape = ModelShape(dtype=torch.float32) if args.decode_fp32 else ModelShape()
-    g = args.decode_grid
+    shape = ModelShape(dtype=torch.float32) if fp32 else ModelShape()
+    g = grid
     prompt = [int(x) for x in torch.randint(0, shape.vocab, (16,), generator=torch.Generator().manual_seed(7))]
-    graphs = not args.decode_eager
-    dec = Decoder(shape, batch=args.decode_batch, grid=(g, g), prompt_len=16, seed=2025, graphs=graphs)
-    # warm-up: a small grid with the same weights (cuBLAS plans, library set-up)
-    Decoder(shape, batch=args.decode_batch, grid=(4, 4), prompt_len=16, seed=2025,
-            target=dec.target_w).generate(prompt)
+    dec = Decoder(shape, batch=batch, grid=(g, g), prompt_len=16, seed=2025, graphs=graphs)
+    # warm-up: the same grid once (cuBLAS plans, library set-up, the CUDA
+    # graph of every tree size the run meets), then the timed run
+    dec.generate(prompt)
     out, st = dec.generate(prompt)
     n = g * g
-    t0 = time.perf_counter()
-    # vanilla greedy decoding in plain torch (bf16 scaled_dot_product_attention, no library call)
-    ref, margins = greedy_decode(shape, dec.target_w, prompt, n, batch=args.decode_batch, return_margins=True,
-                                 graphs=graphs, attn_dtype=torch.bfloat16)
-    torch.cuda.synchronize()
-    t_van = time.perf_counter() - t0
-    same = sum(1 for b in range(args.decode_batch) for x, y in zip(out[b], ref[b]) if x == y)
-    diffs = [next((i for i, (x, y) in enumerate(zip(out[b], ref[b])) if x != y), n) for b in range(args.decode_batch)]
-    first_diff = min(diffs)
-    # the greedy decision there, as a top-2 gap over the logit row's spread (a near tie when tiny)
-    gaps = [margins[b][diffs[b]] for b in range(args.decode_batch) if diffs[b] < n]
-    line = {"metric": "synthetic end-to-end decode tokens/s", "value": st.tokens / st.seconds, "unit": "tokens/s",
+    van = {}
+    greedy_decode(shape, dec.target_w, prompt, n, batch=batch, graphs=graphs, attn_dtype=torch.bfloat16, stats=van)
+    t_van = van["seconds"]
+    choice, margins = greedy_decode(shape, dec.target_w, prompt, n, batch=batch, return_margins=True, graphs=graphs,
+                                    attn_dtype=torch.bfloat16, forced=out)
+    diff = [(b, i) for b in range(batch) for i in range(n) if out[b][i] != choice[b][i]]
+    return {"tokens_per_s": st.tokens / st.seconds, "tau": st.tau, "accepted_draft_tokens": st.accepted,
+            "verify_steps": st.steps, "mean_depth": st.mean_depth, "seconds": st.seconds,
+            "vanilla_greedy_tokens_per_s": batch * n / t_van,
+            "speedup_vs_vanilla": (st.tokens / st.seconds) / (batch * n / t_van),
+            "tokens_differing_from_target_greedy": len(diff), "tokens_checked": batch * n,
+            "max_relative_top2_gap_where_differing": max((margins[b][i] for b, i in diff), default=None),
+            "workload": f"random-init 7B-shape target (32 layers, hidden 4096, 32 heads x 128, SwiGLU 11008, vocab "
+                        f"65536) + one-layer EAGLE-style draft head, {g}x{g} image tokens after a 16-token prompt, "
+                        f"ADT-Tree controller (Anole bounds), greedy, batch {batch}",
+            "dense_dtype": "fp32" if fp32 else "bf16", "launch": "CUDA graph per tree size" if graphs else "eager"}
+
+
+def run_decode(args):
+    """bench.py --decode: one JSON line for the decode loop alone."""
+    d = decode_measure(args.decode_batch, args.decode_grid, args.decode_fp32, not args.decode_eager)
+    line = {"metric": "synthetic end-to-end decode tokens/s", "value": d.pop("tokens_per_s"), "unit": "tokens/s",
             "n_gpus": 1, "higher_is_better": True, "dtype": "bf16", "data": "synthetic (random-init weights)",
-            "config": {"workload": f"random-init 7B-shape target (32 layers, hidden 4096, 32 heads x 128, SwiGLU "
-                                   f"11008, vocab 65536) + one-layer EAGLE-style draft head, {g}x{g} image tokens "
-                                   f"after a 16-token prompt, ADT-Tree controller (Anole bounds), greedy",
-                       "batch": args.decode_batch,
-                       "dense_dtype": "fp32" if args.decode_fp32 else "bf16",
-                       "launch": "CUDA graph per tree size" if graphs else "eager"},
-            "tau": st.tau, "accepted_draft_tokens": st.accepted, "verify_steps": st.steps,
-            "mean_depth": st.mean_depth, "seconds": st.seconds,
-            "vanilla_greedy_tokens_per_s": args.decode_batch * n / t_van,
-            "speedup_vs_vanilla": (st.tokens / st.seconds) / (args.decode_batch * n / t_van),
-            "tokens_equal_to_vanilla_before_first_difference": first_diff, "tokens_equal_total": same,
-            "vanilla_relative_top2_gap_at_first_difference": max(gaps) if gaps else None}
+            "config": {"workload": d.pop("workload"), "batch": args.decode_batch, "dense_dtype": d.pop("dense_dtype"),
+                       "launch": d.pop("launch")}}
+    line.update(d)
     print(json.dumps(line), flush=True)
 
 
@@ -569,6 +637,9 @@ def main():
     ap.add_argument("--decode-grid", type=int, default=48)
     ap.add_argument("--decode-fp32", action="store_true", help="fp32 weights and residual stream in the harness")
     ap.add_argument("--decode-eager", action="store_true", help="no CUDA graphs in the decode loop")
+    ap.add_argument("--no-decode", action="store_true", help="skip the decode-loop measurement of the default run")
+    ap.add_argument("--bench-decode-grid", type=int, default=16,
+                    help="image-token grid side of the decode-loop measurement in the default run")
     args = ap.parse_args()
     if args.decode:
         run_decode(args)
@@ -664,6 +735,10 @@ def main():
         "clocks": r["clocks"],
         "cpu_baseline": cpu,
     }
+    if world == 1 and not args.no_decode and args.workload == "7b":
+        # The end-to-end decode loop (synthetic config C5) at batch 1 and 4,
+        # on a bounded grid so that the default run stays within minutes.
+        line["decode"] = {f"batch{bs}": decode_measure(bs, args.bench_decode_grid) for bs in (1, 4)}
     print(json.dumps(line), flush=True)
     if world > 1:
         import torch

@@ -503,7 +503,7 @@ class DenseModel:
 
 
 def greedy_decode(shape: ModelShape, weights: DecoderWeights, prompt, n_tokens, device="cuda", batch=1,
-                  return_margins=False, graphs=False, attn_dtype=torch.float32, forced=None):
+                  return_margins=False, graphs=False, attn_dtype=torch.float32, forced=None, stats=None):
     """Vanilla greedy decoding with the same target, one token per step,
     through DenseModel: none of the library's entry points (neither its
     attention nor its KV commit) is on this path, so it is an independent
@@ -515,7 +515,9 @@ def greedy_decode(shape: ModelShape, weights: DecoderWeights, prompt, n_tokens, 
     forced (a [batch][n_tokens] token list) teacher-forces the sequence: step
     i still returns the target's greedy choice, but the token fed to step
     i + 1 is forced[b][i], so every position of another decoder's output can
-    be checked against the target's choice given that output's own prefix."""
+    be checked against the target's choice given that output's own prefix.
+    stats (a dict), if given, receives the seconds of the token loop alone
+    (after the prefill and any graph capture)."""
     if not 2 <= len(prompt) <= 257:
         raise ValueError("prompt of 2 .. 257 tokens")
     P = len(prompt)
@@ -548,6 +550,9 @@ def greedy_decode(shape: ModelShape, weights: DecoderWeights, prompt, n_tokens, 
         model.v_cache.copy_(saved[1])
     feed = None if forced is None else torch.tensor(forced, dtype=torch.long, device=dev)
     out, margins = [], []
+    if str(dev).startswith("cuda"):
+        torch.cuda.synchronize()
+    t0 = time.perf_counter()
     for i in range(n_tokens):
         if graph is not None:
             graph.replay()
@@ -559,6 +564,8 @@ def greedy_decode(shape: ModelShape, weights: DecoderWeights, prompt, n_tokens, 
         root.copy_(nxt if feed is None else feed[:, i])
         start += 1
     toks = torch.stack(out, 1).cpu().tolist()
+    if stats is not None:  # (the .cpu() above waited for the device)
+        stats["seconds"] = time.perf_counter() - t0
     if return_margins:
         return toks, torch.stack(margins, 1).cpu().tolist()
     return toks
