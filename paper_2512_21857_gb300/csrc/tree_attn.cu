@@ -33,11 +33,14 @@
 // Every mbarrier wait is bounded; a timeout sets ADT_DEVERR_TIMEOUT.
 //
 // The splits of one (tree, head) form a thread-block cluster (<= 8).  Each
-// split pushes its unnormalised partial rows (O, running max, row sum) into
-// the shared memory of the split that owns those rows, which then merges
-// them locally; with more splits they merge through the workspace.
+// split pushes its partial rows (O, running max, row sum) into the shared
+// memory of the split that owns those rows, which then merges them locally;
+// at D = 128 a row travels as O / l in fp16 with a power-of-two scale (half
+// the bytes of fp32, which the copies between SMs are bound by).  With more
+// splits they merge through the workspace.
 #include <cooperative_groups.h>
 #include <cuda.h>
+#include <cuda_fp16.h>
 
 #include <mutex>
 
@@ -83,7 +86,13 @@ struct Cfg {
   static constexpr int kStageBytes = 2 * kStageTile;     // K tile, then V tile
   static constexpr int kPBytes = 2 * kBlock64;           // 64 query rows x 128 keys
   static constexpr int kStages = D == 128 ? 2 : 4;
-  static constexpr int kRowStride = D + 8;               // fp32 per merged row: D values, m, l, pad
+  // A partial row of the cluster merge, in 32-bit words.  D = 128: D fp16
+  // values (O / l scaled by 2^-e), then m, l (fp32) and e (int32), padded to
+  // 16 bytes; D = 64: D fp32 values (O), m, l, padding (distributed shared
+  // memory moves its rows fast enough that the conversions would cost more
+  // than the halved bytes save).
+  static constexpr bool kHalfRows = D == 128;
+  static constexpr int kRowStride = kHalfRows ? D / 2 + 4 : D + 8;
   static constexpr int kQOff = 0;
   static constexpr int kPOff = kTreeTile;                // Q is 64 rows x D, like a tree tile
   static constexpr int kStageOff = kPOff + 2 * kPBytes;  // the tree unit's K/V go to slot 0
@@ -890,20 +899,66 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (tid == 0)
       sm100::mbar_arrive_expect_tx(sm100::smem_addr(&bars.recv), static_cast<uint32_t>(S * rows_mine * RS * 4));
     if (warp < kSoftmaxWarps) {
+      if constexpr (C::kHalfRows) {
+        // The row normalised by its sum, O / l, goes out in fp16: half the
+        // bytes through distributed shared memory.  It is a convex
+        // combination of V rows, scaled by 2^-e (e from the row's largest
+        // magnitude, over the quad) into [2^14, 2^15): no overflow, and full
+        // fp16 precision relative to that magnitude whatever V's range; the
+        // owner undoes the scale.
 #pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        const int r = half ? rb : ra;
-        if (r < nq) {
-          float* dst = rows_out + r * RS;
-          if (t4 == 0) *reinterpret_cast<float2*>(dst + D) = half ? make_float2(m_rb, l_rb) : make_float2(m_ra, l_ra);
+        for (int half = 0; half < 2; ++half) {
+          const int r = half ? rb : ra;
+          const float l = half ? l_rb : l_ra;
+          const float inv = have_o && l > 0.f ? __fdividef(1.f, l) : 0.f;
+          float amax = 0.f;
 #pragma unroll
-          for (int c = 0; c < kOB; ++c) {
+          for (int c = 0; c < kOB; ++c)
 #pragma unroll
             for (int bk = 0; bk < 8; ++bk)
-              *reinterpret_cast<float2*>(dst + c * 64 + 8 * bk + 2 * t4) =
-                  have_o ? make_float2(__uint_as_float(o[c][4 * bk + 2 * half]),
-                                       __uint_as_float(o[c][4 * bk + 2 * half + 1]))
-                         : make_float2(0.f, 0.f);
+              if (have_o)
+                amax = fmaxf(amax, fmaxf(fabsf(__uint_as_float(o[c][4 * bk + 2 * half])),
+                                         fabsf(__uint_as_float(o[c][4 * bk + 2 * half + 1]))));
+          amax = fmaxf(amax, __shfl_xor_sync(adt::kFullMask, amax, 1));
+          amax = fmaxf(amax, __shfl_xor_sync(adt::kFullMask, amax, 2));
+          amax *= inv;
+          const int ex = static_cast<int>((__float_as_uint(amax) >> 23) & 0xFFu);  // biased exponent
+          const int e = amax > 0.f ? min(max(ex - 127 - 14, -110), 110) : 0;
+          const float sc = inv * __uint_as_float(static_cast<uint32_t>(127 - e) << 23);  // inv * 2^-e
+          if (r < nq) {
+            float* dst = rows_out + r * RS;
+            if (t4 == 0) {
+              *reinterpret_cast<float2*>(dst + D / 2) =
+                  make_float2(have_o ? (half ? m_rb : m_ra) : -INFINITY, have_o ? l : 0.f);
+              reinterpret_cast<int*>(dst)[D / 2 + 2] = e;
+            }
+#pragma unroll
+            for (int c = 0; c < kOB; ++c) {
+#pragma unroll
+              for (int bk = 0; bk < 8; ++bk)
+                reinterpret_cast<__half2*>(dst)[(c * 64 + 8 * bk + 2 * t4) / 2] =
+                    have_o ? __floats2half2_rn(__uint_as_float(o[c][4 * bk + 2 * half]) * sc,
+                                               __uint_as_float(o[c][4 * bk + 2 * half + 1]) * sc)
+                           : __floats2half2_rn(0.f, 0.f);
+            }
+          }
+        }
+      } else {
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          const int r = half ? rb : ra;
+          if (r < nq) {
+            float* dst = rows_out + r * RS;
+            if (t4 == 0) *reinterpret_cast<float2*>(dst + D) = half ? make_float2(m_rb, l_rb) : make_float2(m_ra, l_ra);
+#pragma unroll
+            for (int c = 0; c < kOB; ++c) {
+#pragma unroll
+              for (int bk = 0; bk < 8; ++bk)
+                *reinterpret_cast<float2*>(dst + c * 64 + 8 * bk + 2 * t4) =
+                    have_o ? make_float2(__uint_as_float(o[c][4 * bk + 2 * half]),
+                                         __uint_as_float(o[c][4 * bk + 2 * half + 1]))
+                           : make_float2(0.f, 0.f);
+            }
           }
         }
       }
@@ -929,56 +984,108 @@ __global__ void __launch_bounds__(kThreads, 1)
       adt::raise_error(p.err, ADT_DEVERR_TIMEOUT);
     // This owner has its rows, so the copies it was sent are complete.
     sm100::cluster_arrive_relaxed();
-    // Thread (row i, column group c4) combines the S partials of that row:
-    // weights 2^(m_c - M) l_c / sum.  A thread takes two items per pass and
-    // loads every split's values of both before combining either.
-    // A split without keys sent zeros with m = -inf (weight 0).
-    auto merge_item = [&](int idx, float2 (&ml)[kMaxClusterSplits], float4 (&v)[kMaxClusterSplits]) {
-      const int i = idx / kC4, c4 = idx % kC4;
-      float M = ml[0].x;
-#pragma unroll
-      for (int c = 1; c < kMaxClusterSplits; ++c) M = fmaxf(M, ml[c].x);
-      float lt = 0.f;
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-      for (int c = 0; c < kMaxClusterSplits; ++c) {
-        const float w = ml[c].x == -INFINITY ? 0.f : ex2_approx(ml[c].x - M);
-        lt += w * ml[c].y;
-        acc.x += w * v[c].x;
-        acc.y += w * v[c].y;
-        acc.z += w * v[c].z;
-        acc.w += w * v[c].w;
-      }
-      const float inv = __fdividef(1.f, lt);
-      __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + row0 + r_lo + i) * p.H + h) * D + c4 * 4;
-      uint2 pk;
-      pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
-      pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
-      *reinterpret_cast<uint2*>(dst) = pk;
-      if (c4 == 0 && p.lse) p.lse[static_cast<int64_t>(node0 + row0 + r_lo + i) * p.H + h] = (M + __log2f(lt)) * kLn2;
-    };
-    auto load_item = [&](int idx, float2 (&ml)[kMaxClusterSplits], float4 (&v)[kMaxClusterSplits]) {
-      const int i = idx / kC4, c4 = idx % kC4;
-#pragma unroll
-      for (int c = 0; c < kMaxClusterSplits; ++c) {
-        if (c < S) {
-          const float* row = slots + (c * rows_per + i) * RS;
-          ml[c] = *reinterpret_cast<const float2*>(row + D);
-          v[c] = *reinterpret_cast<const float4*>(row + c4 * 4);
-        } else {
-          ml[c] = make_float2(-INFINITY, 0.f);
-          v[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if constexpr (C::kHalfRows) {
+      // Thread (row i, 8-column group c8) combines the S normalised partials
+      // of that row: weights 2^(m_c - M) l_c / sum (times 2^e_c, the scale the
+      // partial was stored at).  A split without keys sent m = -inf (weight 0).
+      constexpr int kC8 = D / 8;
+      for (int idx = tid; idx < rows_mine * kC8; idx += kThreads) {
+        const int i = idx / kC8, c8 = idx % kC8;
+        float2 ml[kMaxClusterSplits];
+        int ec[kMaxClusterSplits];
+        uint4 v[kMaxClusterSplits];
+  #pragma unroll
+        for (int c = 0; c < kMaxClusterSplits; ++c) {
+          if (c < S) {
+            const float* row = slots + (c * rows_per + i) * RS;
+            ml[c] = *reinterpret_cast<const float2*>(row + D / 2);
+            ec[c] = reinterpret_cast<const int*>(row)[D / 2 + 2];
+            v[c] = *reinterpret_cast<const uint4*>(row + c8 * 4);
+          }
         }
+        float M = -INFINITY;
+  #pragma unroll
+        for (int c = 0; c < kMaxClusterSplits; ++c)
+          if (c < S) M = fmaxf(M, ml[c].x);
+        float lt = 0.f;
+        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  #pragma unroll
+        for (int c = 0; c < kMaxClusterSplits; ++c) {
+          if (c < S) {
+            const float w = ml[c].x == -INFINITY ? 0.f : ex2_approx(ml[c].x - M) * ml[c].y;
+            lt += w;
+            const float ws = w * __uint_as_float(static_cast<uint32_t>(127 + ec[c]) << 23);  // w * 2^e_c
+            const __half2* hv = reinterpret_cast<const __half2*>(&v[c]);
+  #pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float2 f = __half22float2(hv[e]);
+              acc[2 * e] += ws * f.x;
+              acc[2 * e + 1] += ws * f.y;
+            }
+          }
+        }
+        const float inv = __fdividef(1.f, lt);
+        __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + row0 + r_lo + i) * p.H + h) * D + c8 * 8;
+        uint4 pk;
+        pk.x = pack_bf16x2(acc[0] * inv, acc[1] * inv);
+        pk.y = pack_bf16x2(acc[2] * inv, acc[3] * inv);
+        pk.z = pack_bf16x2(acc[4] * inv, acc[5] * inv);
+        pk.w = pack_bf16x2(acc[6] * inv, acc[7] * inv);
+        *reinterpret_cast<uint4*>(dst) = pk;
+        if (c8 == 0 && p.lse) p.lse[static_cast<int64_t>(node0 + row0 + r_lo + i) * p.H + h] = (M + __log2f(lt)) * kLn2;
       }
-    };
-    for (int idx = tid; idx < rows_mine * kC4; idx += 2 * kThreads) {
-      float2 ml0[kMaxClusterSplits], ml1[kMaxClusterSplits];
-      float4 v0[kMaxClusterSplits], v1[kMaxClusterSplits];
-      const bool two = idx + kThreads < rows_mine * kC4;
-      load_item(idx, ml0, v0);
-      if (two) load_item(idx + kThreads, ml1, v1);
-      merge_item(idx, ml0, v0);
-      if (two) merge_item(idx + kThreads, ml1, v1);
+    } else {
+      // Thread (row i, column group c4) combines the S partials of that row:
+      // weights 2^(m_c - M) l_c / sum.  A thread takes two items per pass and
+      // loads every split's values of both before combining either.
+      // A split without keys sent zeros with m = -inf (weight 0).
+      auto merge_item = [&](int idx, float2 (&ml)[kMaxClusterSplits], float4 (&v)[kMaxClusterSplits]) {
+        const int i = idx / kC4, c4 = idx % kC4;
+        float M = ml[0].x;
+  #pragma unroll
+        for (int c = 1; c < kMaxClusterSplits; ++c) M = fmaxf(M, ml[c].x);
+        float lt = 0.f;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  #pragma unroll
+        for (int c = 0; c < kMaxClusterSplits; ++c) {
+          const float w = ml[c].x == -INFINITY ? 0.f : ex2_approx(ml[c].x - M);
+          lt += w * ml[c].y;
+          acc.x += w * v[c].x;
+          acc.y += w * v[c].y;
+          acc.z += w * v[c].z;
+          acc.w += w * v[c].w;
+        }
+        const float inv = __fdividef(1.f, lt);
+        __nv_bfloat16* dst = p.out + (static_cast<int64_t>(node0 + row0 + r_lo + i) * p.H + h) * D + c4 * 4;
+        uint2 pk;
+        pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+        pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+        *reinterpret_cast<uint2*>(dst) = pk;
+        if (c4 == 0 && p.lse) p.lse[static_cast<int64_t>(node0 + row0 + r_lo + i) * p.H + h] = (M + __log2f(lt)) * kLn2;
+      };
+      auto load_item = [&](int idx, float2 (&ml)[kMaxClusterSplits], float4 (&v)[kMaxClusterSplits]) {
+        const int i = idx / kC4, c4 = idx % kC4;
+  #pragma unroll
+        for (int c = 0; c < kMaxClusterSplits; ++c) {
+          if (c < S) {
+            const float* row = slots + (c * rows_per + i) * RS;
+            ml[c] = *reinterpret_cast<const float2*>(row + D);
+            v[c] = *reinterpret_cast<const float4*>(row + c4 * 4);
+          } else {
+            ml[c] = make_float2(-INFINITY, 0.f);
+            v[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+        }
+      };
+      for (int idx = tid; idx < rows_mine * kC4; idx += 2 * kThreads) {
+        float2 ml0[kMaxClusterSplits], ml1[kMaxClusterSplits];
+        float4 v0[kMaxClusterSplits], v1[kMaxClusterSplits];
+        const bool two = idx + kThreads < rows_mine * kC4;
+        load_item(idx, ml0, v0);
+        if (two) load_item(idx + kThreads, ml1, v1);
+        merge_item(idx, ml0, v0);
+        if (two) merge_item(idx + kThreads, ml1, v1);
+      }
     }
     // Every owner has its rows: this CTA's outgoing copies are complete.
     sm100::cluster_wait_acquire();

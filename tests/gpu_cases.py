@@ -11,8 +11,14 @@ import oracle
 from paper_2512_21857_gb300 import binding as B
 from paper_2512_21857_gb300 import synth
 
-ATOL = 1e-2      # attention: max |gpu - oracle| elementwise
-NORM_RTOL = 2e-2  # attention: max |gpu - oracle| / max |oracle|
+# Attention: |gpu - oracle| <= ATOL + OUT_RTOL |oracle| elementwise, and
+# max |gpu - oracle| / max |oracle| <= NORM_RTOL.  ATOL covers the outputs
+# of long prefixes (|o| ~ 0.02-0.1); the output is bf16, whose rounding alone
+# is up to half an ulp, 2^-9 |o|, which exceeds ATOL / 2 once |o| > 2.5 (rows
+# that see few keys, short prefixes): OUT_RTOL adds that half ulp.
+ATOL = 1e-2
+OUT_RTOL = 2.0 ** -9
+NORM_RTOL = 2e-2
 # lse: the log of the normaliser the kernel applies, the sum of the
 # probabilities as rounded to bf16 for the PV product; each rounding is
 # within a relative 2^-9, so the sum (and its log) is within 2^-9 of the
@@ -76,7 +82,8 @@ class AttnCase:
 
 def assert_attention_close(got, ref):
     err = np.abs(got - ref)
-    assert err.max() <= ATOL, f"max abs err {err.max():.3e}"
+    excess = err - (ATOL + OUT_RTOL * np.abs(ref))
+    assert excess.max() <= 0, f"max abs err {err.max():.3e}, max excess over the bound {excess.max():.3e}"
     assert err.max() / max(np.abs(ref).max(), 1e-30) <= NORM_RTOL, "normwise error"
 
 
