@@ -202,3 +202,40 @@ def test_rerank_matches_oracle(C, n, flat):
     ref = oracle.tree_rerank(tok, sc, par, 7, n)
     for key in res:
         assert np.array_equal(res[key].cpu().numpy(), ref[key]), key
+
+
+def test_expand_masked_vocabulary_few_finite_values_per_cta():
+    """Logits -inf (a masked vocabulary) except one or two per eighth of the
+    row: every CTA of the row holds fewer than k finite values, so its bound
+    falls to -inf and the overflow path ranks its whole share; the k
+    children are the row's finite logits, best first."""
+    V, F, k = 65536, 2, 8
+    g = np.random.default_rng(3)
+    logits = np.full((F, V), -np.inf, np.float32)
+    for r in range(F):
+        for c in range(8):
+            pos = g.choice(8192, size=1 + (c % 2), replace=False) + 8192 * c
+            logits[r, pos] = g.normal(0.0, 3.0, size=len(pos)).astype(np.float32)
+    fscore = np.array([-0.5, -1.5], np.float32)
+    got, _ = run_expand(logits, fscore, None, k, 8)
+    ref = oracle.tree_expand(logits, fscore, k, 8)
+    assert np.isfinite(ref["child_score"]).all()
+    check_expand(got, ref, 8)
+
+
+def test_expand_finite_values_held_by_one_thread():
+    """The only finite logits sit where one thread holds them (indices 0-3
+    and 1024 of an 1100-wide row, one CTA): fewer than k lanes have a finite
+    maximum, the bound is -inf, and every logit of the share is a candidate
+    without overflowing the candidate buffer."""
+    F, k = 3, 5
+    for V in (1100,):
+        logits = np.full((F, V), -np.inf, np.float32)
+        g = np.random.default_rng(V)
+        for r in range(F):
+            logits[r, [0, 1, 2, 3, 1024]] = g.normal(0.0, 2.0, size=5).astype(np.float32)
+        fscore = np.zeros(F, np.float32)
+        got, _ = run_expand(logits, fscore, None, k, 5)
+        ref = oracle.tree_expand(logits, fscore, k, 5)
+        assert np.isfinite(ref["child_score"]).all()
+        check_expand(got, ref, 5)
