@@ -189,3 +189,27 @@ def test_value_range_extremes(scale):
     assert np.isfinite(got).all()
     assert_attention_close(got / scale, ref / scale)
     assert np.abs(lse - ref_lse).max() < LSE_ATOL
+
+
+def test_zero_and_mixed_magnitude_values():
+    """V all zero (every partial row's largest magnitude is 0: outputs
+    exactly 0), then V rows whose magnitudes differ by 2^40 between heads and
+    between halves of the prefix, so that the splits of one head stage rows
+    at very different scales: the cluster merge must combine them by their
+    weights alone.  The 7B launch shape (4 splits per head)."""
+    import torch
+    case = AttnCase([64], [2400], 32, 32, 128, seed=32, lmax=2400 + 64)
+    vc, vt = case.vc.clone(), case.vt.clone()
+    case.vc = torch.zeros_like(vc)
+    case.vt = torch.zeros_like(vt)
+    got, _, _ = case.run_gpu(max_kv=2400 + 64)
+    assert not got.any()
+    scale_h = (2.0 ** (torch.arange(32) % 5 * 10 - 20)).view(1, 32, 1, 1)   # per head: 2^-20 .. 2^20
+    scale_pos = torch.where(torch.arange(2400 + 64) < 1200, 1.0, 2.0 ** -20).view(1, 1, -1, 1)
+    case.vc = (vc.float() * scale_h * scale_pos).to(torch.bfloat16)
+    case.vt = (vt.float() * scale_h.view(1, 32, 1)).to(torch.bfloat16)
+    got, _, _ = case.run_gpu(max_kv=2400 + 64)
+    ref, _ = case.run_oracle()
+    s = scale_h.view(32, 1).numpy().astype(np.float64)
+    for h in range(32):
+        assert_attention_close(got[:, h] / s[h], ref[:, h] / s[h])
