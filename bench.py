@@ -594,6 +594,7 @@ def decode_measure(batch, grid, fp32=False, graphs=True):
     diff = [(b, i) for b in range(batch) for i in range(n) if out[b][i] != choice[b][i]]
     attn = decode_verify_attention(dec, prompt_len=16, n=n)
     return {"tokens_per_s": st.tokens / st.seconds, "tau": st.tau, "accepted_draft_tokens": st.accepted,
+            "accepted_length_histogram": {str(k): v for k, v in sorted(st.accept_hist.items())},
             "verify_steps": st.steps, "mean_depth": st.mean_depth, "seconds": st.seconds,
             "vanilla_greedy_tokens_per_s": batch * n / t_van,
             "speedup_vs_vanilla": (st.tokens / st.seconds) / (batch * n / t_van),

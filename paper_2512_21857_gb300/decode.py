@@ -28,7 +28,7 @@ from __future__ import annotations
 
 import math
 import time
-from dataclasses import dataclass
+from dataclasses import dataclass, field
 
 import torch
 
@@ -202,6 +202,7 @@ class DecodeStats:
     tokens: int = 0
     steps: int = 0
     accepted: int = 0          # accepted draft tokens (the bonus tokens not counted)
+    accept_hist: dict = field(default_factory=dict)  # accepted length -> (image, step) count
     seconds: float = 0.0
     depth_sum: int = 0
     batch: int = 1
@@ -435,6 +436,7 @@ class Decoder:
             for b in range(self.batch):
                 out[b] += emitted[b]
                 stats.accepted += alen[b]
+                stats.accept_hist[alen[b]] = stats.accept_hist.get(alen[b], 0) + 1
         torch.cuda.synchronize()
         stats.seconds = time.perf_counter() - t0
         stats.tokens = sum(len(o) for o in out)
