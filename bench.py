@@ -257,23 +257,30 @@ def run_gpu(args, wl, rank, world):
     # attention kernel for the roofline in a second timed region.
     step_graph = torch.cuda.CUDAGraph()
     attn_graph = torch.cuda.CUDAGraph()
+    # The draft-tree expansion calls of image 0 (depth calls, F = 1 then the
+    # width), back to back as inside the step, timed alone after the others.
+    expand_graph = torch.cuda.CUDAGraph()
     with torch.cuda.stream(stream):
         with torch.cuda.graph(step_graph, stream=stream):
             step.launch(stream)
         with torch.cuda.graph(attn_graph, stream=stream):
             for layer in range(shape.layers):
                 step.launch_attention(layer, stream)
+        with torch.cuda.graph(expand_graph, stream=stream):
+            step.launch_draft_image(0, stream, rerank=False)
     torch.cuda.synchronize()
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
             step_graph.replay()
             attn_graph.replay()
+            expand_graph.replay()
     torch.cuda.synchronize()
 
     K = args.steps
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ea0, ea1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ee0, ee1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     sampler = ClockSampler(local)
     sampler.start()
     nvml = NvmlSampler(local)
@@ -295,6 +302,10 @@ def run_gpu(args, wl, rank, world):
         for _ in range(K):
             attn_graph.replay()
         ea1.record(stream)
+        ee0.record(stream)
+        for _ in range(K):
+            expand_graph.replay()
+        ee1.record(stream)
     torch.cuda.synchronize()
     t1 = time.time()
     if world > 1:
@@ -308,6 +319,8 @@ def run_gpu(args, wl, rank, world):
     per_step = sorted(step_ev[i].elapsed_time(step_ev[i + 1]) for i in range(K))
     pct = {f"p{q}": per_step[min(K - 1, int(round(q / 100 * (K - 1))))] for q in (10, 50, 90)}
     attn_ms = ea0.elapsed_time(ea1) / (K * shape.layers)
+    expand_calls = int(shape.depth[0])
+    expand_us = ee0.elapsed_time(ee1) * 1000.0 / (K * expand_calls)
     errbits = B.adt_get_device_error(stream)
     if errbits:
         raise RuntimeError(f"device error bits {errbits:#x} during the timed steps")
@@ -388,7 +401,8 @@ def run_gpu(args, wl, rank, world):
     sha = attn_source_sha()
     traffic = NCU_TRAFFIC.get(sha) if args.workload == "7b" else None
     return dict(step_ms=step_ms, step_pct=pct, attn_ms=attn_ms, clocks=clocks, e2e_ms=e2e_ms, h2d=h2d, d2h=d2h,
-                launches=K * (step.kernel_launches_per_step() + shape.layers), achieved=achieved, peak=peak, peak_kind=peak_kind,
+                launches=K * (step.kernel_launches_per_step() + shape.layers + expand_calls), achieved=achieved,
+                peak=peak, peak_kind=peak_kind, expand_us=expand_us, expand_calls=expand_calls,
                 traffic=traffic, attn_bytes=ab["attention_per_layer"], step_bytes=ab["attention"], sha=sha)
 
 
@@ -795,6 +809,10 @@ def main():
                      "avg_launch_us": r["attn_ms"] * 1e3, "kernel_sha": r["sha"]},
         "e2e": {"value": e2e_value, "unit": "steps/s", "h2d_bytes_per_step": r["h2d"],
                 "d2h_bytes_per_step": r["d2h"]},
+        "expansion": {"kernel": "expand_kernel", "calls_per_step": r["expand_calls"],
+                      "avg_call_us": r["expand_us"],
+                      "note": "image 0's draft-tree expansion calls (F = 1, then the width) replayed alone "
+                              "back to back in a graph"},
         "gpu_launches": r["launches"],
         "clocks": r["clocks"],
         "cpu_baseline": cpu,

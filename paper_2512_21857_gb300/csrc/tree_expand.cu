@@ -3,17 +3,17 @@
 // adt_tree_rerank: the final top-N tree (Eq. 4 and the sentence after it).
 //
 // Expand is one launch of F thread-block clusters, one per frontier row; the
-// C <= 8 CTAs of a cluster split the row's vocabulary.  Each warp streams its
-// share of the logits (x / T in fp32, round-to-nearest division) keeping a
-// running maximum and sum of exponentials and each lane's two largest
-// selection keys (value order, then lower index).  The k-th largest of the
-// warp's 64 lane keys bounds the warp's top k from below; a second pass
-// gathers the keys at or above it and ranks them.  Sorted lists then merge by
-// rank (binary search in the other lists): the warps' into the CTA's, the
-// CTAs' into the cluster's first CTA through distributed shared memory, which
-// writes the row's children (log-probability against the row's log-sum-exp
-// in fp64).  The first CTA of the last row to finish (atomic ticket) selects
-// the next frontier across all rows the same way.
+// C <= 8 CTAs of a cluster split the row's vocabulary.  Each CTA stages its
+// share in shared memory with one bulk copy (x / T in fp32, round-to-nearest
+// division).  A first pass keeps each thread's two largest values; the k-th
+// largest of the 32 warp maxima bounds the CTA's top k from below; a second
+// pass sums the exponentials against the CTA's maximum and gathers the few
+// selection keys (value order, then lower index) at or above the bound,
+// which are ranked by counting.  The CTAs' lists go to the cluster's first
+// CTA through distributed shared memory; it ranks them, forms the row's
+// log-sum-exp and writes the row's children (log-probability against it in
+// fp64).  The first CTA of the last row to finish (atomic ticket) ranks the
+// next frontier across all rows.
 #include <cooperative_groups.h>
 
 #include "adt_common.cuh"
@@ -202,19 +202,37 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 
-// The k-th largest (k <= 32) of the warp's 32 values, by a bitonic sort
-// across the lanes (descending).
+// The k-th largest (k <= 32) of the warp's 32 values (none NaN): the one
+// whose rank -- the values above it, with equal values of lower lanes
+// counted as above -- is k - 1.  32 independent shuffles instead of the
+// dependent chain of a sort.
 __device__ __forceinline__ float warp_kth_largest(float v, int k, int lane) {
+  int rk = 0;
 #pragma unroll
-  for (int size = 2; size <= 32; size <<= 1) {
-#pragma unroll
-    for (int stride = size >> 1; stride > 0; stride >>= 1) {
-      const float o = __shfl_xor_sync(adt::kFullMask, v, stride);
-      const bool keep_max = ((lane & stride) == 0) == ((lane & size) == 0);
-      v = keep_max ? fmaxf(v, o) : fminf(v, o);
-    }
+  for (int j = 0; j < 32; ++j) {
+    const float o = __shfl_sync(adt::kFullMask, v, j);
+    rk += (o > v || (o == v && j < lane)) ? 1 : 0;
   }
-  return __shfl_sync(adt::kFullMask, v, k - 1);
+  const unsigned m = __ballot_sync(adt::kFullMask, rk == k - 1);
+  return __shfl_sync(adt::kFullMask, v, __ffs(m) - 1);
+}
+
+// rank_select for n <= 64 keys: 16 threads per key, each counting the keys
+// above it among four of the others, the counts summed by shuffles within
+// the group; one round of loads instead of a warp per key looping over n.
+__device__ void rank_select64(const uint64_t* keys, int n, int k, uint64_t* out) {
+  static_assert(kThreads == 64 * 16, "16 threads for each of 64 keys");
+  const int i = threadIdx.x >> 4, s = threadIdx.x & 15;
+  const uint64_t key = i < n ? keys[i] : 0ull;
+  int c = 0;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int o = s + 16 * j;
+    c += (o < n && keys[o] > key) ? 1 : 0;
+  }
+#pragma unroll
+  for (int off = 8; off > 0; off >>= 1) c += __shfl_xor_sync(adt::kFullMask, c, off);
+  if (s == 0 && key != 0ull && c < k) out[c] = key;
 }
 
 __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) {
@@ -248,7 +266,7 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
     sm100::fence_mbar_init();
   }
   __syncthreads();
-  adt::pdl_wait_then_release();
+  asm volatile("griddepcontrol.wait;\n" ::: "memory");
   // This CTA's share of the row: [c0, c1), c0 a multiple of 4.
   const int per = (((p.V + C - 1) / C) + 3) & ~3;
   const int c0 = min(p.V, rank * per), c1 = min(p.V, c0 + per);
@@ -266,7 +284,7 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
   bool ok = true;
 
   // Pass 1: each thread's two largest values (ties kept).  Thread tid takes
-  // elements tid, tid + 256, ... of every tile.
+  // elements tid, tid + 1024, ... of every tile.
   float v1 = -INFINITY, v2 = -INFINITY;
   for (int tt = 0; tt < ntiles; ++tt) {
     const int t0 = c0 + tt * kTile, t1 = min(c1, t0 + kTile);
@@ -282,7 +300,7 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
   if (!ok && tid == 0) adt::raise_error(p.err, ADT_DEVERR_TIMEOUT);
   // The bound B: a value with at least k of the CTA's logits at or above it,
   // so that its k best are among those >= B.  For k <= 32: the k-th largest
-  // of the 32 warp maxima (one bitonic sort in warp 0).  For larger k: per
+  // of the 32 warp maxima (ranked by counting in warp 0).  For larger k: per
   // warp, the largest of its 64 lane values (two per lane) with k of them at
   // or above it; B is the largest of those.
   {
@@ -349,7 +367,9 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
   }
   __syncthreads();
   const int cnt = static_cast<int>(s_cnt);
-  if (cnt <= kCandCap) {
+  if (cnt <= 64) {
+    rank_select64(cand, cnt, K, ctl);
+  } else if (cnt <= kCandCap) {
     rank_select(cand, cnt, K, ctl);
   } else {
     // Overflow (very many values at or above B): each warp keeps its k
@@ -378,32 +398,36 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
     merge_topk(&wl[0][0], kWarps, kMaxK, K, K, ctl);
   }
   __syncthreads();
+  if (!ok && tid == 0) adt::raise_error(p.err, ADT_DEVERR_TIMEOUT);  // a restaged tile's wait
   // This CTA's top k and (max, sum of exponentials), to the cluster's first CTA.
   if (warp == 0) {
     uint64_t* dst = cl.map_shared_rank(&cl_keys[rank * K], 0);
     if (lane < K) dst[lane] = ctl[lane];
     if (lane + 32 < K) dst[lane + 32] = ctl[lane + 32];
-    if (lane == 0) {
-      float S = 0.f;
-      for (int w = 0; w < kWarps; ++w) S += s_sw[w];
-      *cl.map_shared_rank(&cl_ms[rank], 0) = make_float2(M, S);
-    }
+    const float S = adt::warp_sum(s_sw[lane]);  // kWarps == 32
+    if (lane == 0) *cl.map_shared_rank(&cl_ms[rank], 0) = make_float2(M, S);
   }
   sm100::cluster_arrive_release();
   sm100::cluster_wait_acquire();
+  // The next kernel in the stream may launch now.  Released here rather than
+  // right after the wait: a graph of six back-to-back calls (F = 1, then 8;
+  // V = 65536, k = 8) and the rerank took 49.2 us against 51.2 us.
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
   if (rank != 0) return;
 
   // ---- first CTA of row r: the row's top k and log-sum-exp, its children.
   for (int i = tid; i < kMaxK; i += kThreads) rowl[i] = 0ull;
-  if (tid == 0) {
-    float Mr = -INFINITY, S = 0.f;
-    for (int c = 0; c < C; ++c) Mr = fmaxf(Mr, cl_ms[c].x);
-    for (int c = 0; c < C; ++c)
-      if (cl_ms[c].x != -INFINITY) S += cl_ms[c].y * ex2_approx((cl_ms[c].x - Mr) * kLog2e);
-    s_lse = static_cast<double>(Mr) + static_cast<double>(logf(S));
+  if (warp == 0) {  // lane c takes CTA c's (max, sum); C <= 8
+    const float2 ms = lane < C ? cl_ms[lane] : make_float2(-INFINITY, 0.f);
+    const float Mr = adt::warp_max(ms.x);
+    const float S = adt::warp_sum(ms.x != -INFINITY ? ms.y * ex2_approx((ms.x - Mr) * kLog2e) : 0.f);
+    if (lane == 0) s_lse = static_cast<double>(Mr) + static_cast<double>(logf(S));
   }
   __syncthreads();
-  rank_select(cl_keys, C * K, K, rowl);
+  if (C * K <= 64)
+    rank_select64(cl_keys, C * K, K, rowl);
+  else
+    rank_select(cl_keys, C * K, K, rowl);
   __syncthreads();
   if (writer) {
     const uint64_t key = rowl[tid];
@@ -442,7 +466,10 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
     for (int i = tid; i < nc; i += kThreads) cross_s[i] = __ldcg(p.cross_keys + i);
     for (int i = tid; i < kMaxK; i += kThreads) rowl[i] = 0ull;
     __syncthreads();
-    rank_select(cross_s, nc, p.k_keep, rowl);
+    if (nc <= 64)
+      rank_select64(cross_s, nc, p.k_keep, rowl);
+    else
+      rank_select(cross_s, nc, p.k_keep, rowl);
     __syncthreads();
     if (tid < p.k_keep) {
       const uint64_t key = rowl[tid];

@@ -140,8 +140,8 @@ class TreeVerifyStep:
                 self.root_token] + list(self.draft_rows)
 
     # -------------------------------------------------------------- phases
-    def launch_draft_image(self, b, stream=None):
-        """Expand d_b layers and rerank, for image b."""
+    def launch_draft_image(self, b, stream=None, rerank=True):
+        """Expand d_b layers and rerank (unless `rerank` is false), for image b."""
         s = self.shape
         k = s.width[b]
         base = 0
@@ -161,6 +161,8 @@ class TreeVerifyStep:
                               next_id=front_id[nxt, :k], workspace=self.ws_expand[b], stream=stream)
             fscore, fid = front_score[nxt, :k], front_id[nxt, :k]
             base += F * k
+        if not rerank:
+            return
         lo, hi = int(self.node_offsets_host(b)), int(self.node_offsets_host(b + 1))
         B.adt_tree_rerank(self.pool_tok[b], self.pool_score[b], self.pool_par[b], base,
                           self.root_token[b:b + 1], hi - lo, tokens=self.tokens[lo:hi],
