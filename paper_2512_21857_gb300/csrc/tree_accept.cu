@@ -418,7 +418,47 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
     if (p.mode == ADT_ACCEPT_GREEDY) {
       float bv = -INFINITY;
       int bi = 0x7fffffff;
-      for (int i = tid; i < cnt; i += kThreads) {
+      // 16-byte loads (the row start and lo are multiples of 4 floats), a
+      // thread's kU loads all issued before any value is compared.
+      constexpr int kU = 4;
+      const int c4 = cnt >> 2;
+      const float4* t4 = reinterpret_cast<const float4*>(trow + lo);
+      const float4* u4 = trow_u ? reinterpret_cast<const float4*>(trow_u + lo) : nullptr;
+      for (int g0 = tid; g0 < c4; g0 += kU * kThreads) {
+        float4 x[kU];
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+          const int g = g0 + u * kThreads;
+          x[u] = g < c4 ? __ldg(t4 + g) : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+        }
+        if (u4) {
+#pragma unroll
+          for (int u = 0; u < kU; ++u) {
+            const int g = g0 + u * kThreads;
+            if (g < c4) {
+              const float4 y = __ldg(u4 + g);
+              x[u].x = adt::cfg_combine(x[u].x, y.x, p.cfg);
+              x[u].y = adt::cfg_combine(x[u].y, y.y, p.cfg);
+              x[u].z = adt::cfg_combine(x[u].z, y.z, p.cfg);
+              x[u].w = adt::cfg_combine(x[u].w, y.w, p.cfg);
+            }
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+          const int g = g0 + u * kThreads;
+          if (g >= c4) continue;
+          const int i = lo + 4 * g;
+          const float e[4] = {x[u].x, x[u].y, x[u].z, x[u].w};
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (better(e[j], i + j, bv, bi)) {
+              bv = e[j];
+              bi = i + j;
+            }
+        }
+      }
+      for (int i = 4 * c4 + tid; i < cnt; i += kThreads) {  // the slice's last (V % 4) values
         float x = __ldg(trow + lo + i);
         if (trow_u) x = adt::cfg_combine(x, __ldg(trow_u + lo + i), p.cfg);
         if (better(x, lo + i, bv, bi)) {
