@@ -48,7 +48,7 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
   } while (0)
 
 // Launch attribute that allows a kernel to overlap the tail of the previous
-// one (its device code calls pdl_wait_then_release before touching memory).
+// one (its device code executes griddepcontrol.wait before touching memory).
 inline cudaLaunchAttribute pdl_attribute() {
   cudaLaunchAttribute a;
   a.id = cudaLaunchAttributeProgrammaticStreamSerialization;
