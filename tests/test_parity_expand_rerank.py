@@ -239,3 +239,24 @@ def test_expand_finite_values_held_by_one_thread():
         ref = oracle.tree_expand(logits, fscore, k, 5)
         assert np.isfinite(ref["child_score"]).all()
         check_expand(got, ref, 5)
+
+
+@pytest.mark.parametrize("n_top", [64, 65, 200, 1024])
+def test_expand_many_values_at_the_bound(n_top):
+    """n_top copies of the row's largest value spread over one CTA's eighth
+    of the row: at least k of that CTA's warp maxima are that value, so its
+    bound equals it and exactly n_top values are candidates.  Up to 64 they
+    are ranked by groups of 16 threads, beyond that by a warp per key (1024:
+    the candidate buffer's capacity).  The row's children are the k copies
+    of lowest index."""
+    V, F, k = 65536, 2, 8
+    g = np.random.default_rng(n_top)
+    logits = g.normal(0.0, 1.0, size=(F, V)).astype(np.float32)
+    pos = np.sort(g.choice(8192, size=n_top, replace=False)) + 8192 * 3
+    assert len(set((pos % 1024) // 32)) >= k  # copies in at least k warps of that CTA
+    logits[0, pos] = np.float32(7.0)
+    fscore = np.array([-1.0, -0.25], np.float32)
+    got, _ = run_expand(logits, fscore, None, k, 8)
+    ref = oracle.tree_expand(logits, fscore, k, 8)
+    assert got["child_token"][:k].tolist() == pos[:k].tolist()
+    check_expand(got, ref, 8)
