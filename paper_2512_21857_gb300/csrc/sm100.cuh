@@ -151,8 +151,6 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;\n" ::: "memory"); }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;\n" ::: "memory"); }
 
-// 32 lanes x 32 bit, 16 consecutive columns: thread t of the warp receives
-// columns [col, col + 16) of lane (warp quadrant base + t).
 // Instruction descriptor of kind::f16 with bf16 A and B, fp32 D.
 // a_mn_major / b_mn_major: 1 if that operand is stored MN-major.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, int a_mn_major, int b_mn_major) {
