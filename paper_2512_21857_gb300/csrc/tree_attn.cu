@@ -14,8 +14,8 @@
 // loaded with Q), then its prefix chunks.
 //
 // Warp roles inside a CTA (256 threads; one thread of each of warps 4-7):
-//   warp 4    TMA tensor loads of prefix K (64 x 64 boxes, 128-byte swizzle)
-//             into a ring of 128-key stages;
+//   warp 4    TMA tensor loads of prefix K (boxes of 128 keys x 64 columns,
+//             128-byte swizzle) into a ring of 128-key stages;
 //   warp 5    tcgen05.mma S = Q K^T into one of two tensor-memory tiles
 //             (M = 64 queries, N = 128 keys), back to back (softmax warp 0
 //             frees each K tile once it sees its S product done);
