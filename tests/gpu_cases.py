@@ -40,6 +40,16 @@ def f32(x, dev="cuda"):
     return torch.as_tensor(np.asarray(x, dtype=np.float32), device=dev)
 
 
+def f32_rows(x, dev="cuda"):
+    """A [rows][V] fp32 array on the device with its rows padded to a multiple
+    of 4 floats (the row stride the ABI requires); the [:, :V] view."""
+    x = np.asarray(x, dtype=np.float32)
+    ld = (x.shape[1] + 3) // 4 * 4
+    t = torch.zeros((x.shape[0], ld), dtype=torch.float32, device=dev)
+    t[:, :x.shape[1]] = torch.as_tensor(x, device=dev)
+    return t[:, :x.shape[1]]
+
+
 class AttnCase:
     """Inputs of one adt_tree_attn call: B trees of the given sizes, prefix
     lengths, heads and head dim."""
@@ -145,7 +155,7 @@ def run_accept_gpu(target, draft, tb, mode, ua=None, us=None, temperature=1.0, m
     path = torch.empty((Bn, max_path), dtype=torch.int32, device=dev)
     alen = torch.empty(Bn, dtype=torch.int32, device=dev)
     bonus = torch.empty(Bn, dtype=torch.int32, device=dev)
-    B.adt_tree_accept(f32(target), None if draft is None else f32(draft), i32(tb.tokens), i32(tb.parents),
+    B.adt_tree_accept(f32_rows(target), None if draft is None else f32_rows(draft), i32(tb.tokens), i32(tb.parents),
                       i32(tb.node_offsets), B=Bn, V=V, max_nodes=int(sizes.max()), mode=mode,
                       u_accept=None if ua is None else f32(ua), u_sample=None if us is None else f32(us),
                       temperature=temperature, path=path, max_path=max_path, accept_len=alen, bonus_token=bonus,

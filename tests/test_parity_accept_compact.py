@@ -57,7 +57,7 @@ def compare(tb, res, path, alen, bonus):
 
 
 @pytest.mark.parametrize("sizes,V", [([26], 16384), ([64], 65536), ([64, 1, 33, 7, 64, 12, 50, 20], 65536),
-                                     ([5], 100), ([3, 9], 262144)])
+                                     ([5], 100), ([3, 9], 262144), ([26, 9], 4099), ([12, 30], 65537)])
 @pytest.mark.parametrize("sigma", [None, 0.3])
 def test_greedy_matches_oracle(sizes, V, sigma):
     seed = sum(sizes) + V
@@ -284,3 +284,31 @@ def test_compact_inplace_rejects_bad_trees():
     assert bits & B.DEVERR_KV_RANGE and bits & B.DEVERR_BAD_PATH
     assert gl.tolist() == [9, 2]
     assert torch.equal(gk, kc) and torch.equal(gv, vc)
+
+
+def test_greedy_ties_take_the_lowest_index():
+    """Every target row holds its largest value several times: in the same
+    16-byte group, in different groups of one thread, in different threads
+    and in different vocabulary slices (CTAs).  The walk's argmax is the
+    lowest of those indices, as the oracle's; a child carrying a later copy
+    is not accepted."""
+    V = 65536
+    tb = synth.tree_batch([20], V, 5)
+    g = np.random.default_rng(5)
+    target = g.normal(0.0, 1.0, size=(20, V)).astype(np.float32)
+    for v in range(20):
+        copies = sorted(g.choice(V, size=6, replace=False).tolist() + [4 * (v + 3) + 1, 4 * (v + 3) + 2])
+        target[v, copies] = np.float32(9.0)
+    # the root's first child carries the root row's lowest copy: accepted;
+    # its first child carries a later copy of that node's row: rejected
+    kids0 = [i for i in range(20) if tb.parents[i] == 0]
+    low0 = int(np.flatnonzero(target[0] == 9.0)[0])
+    tb.tokens[kids0[0]] = low0
+    c = kids0[0]
+    kids1 = [i for i in range(20) if tb.parents[i] == c]
+    if kids1:
+        tb.tokens[kids1[0]] = int(np.flatnonzero(target[c] == 9.0)[1])
+    res = oracle.tree_accept(target, None, tb.tokens, tb.parents, tb.node_offsets, oracle.ACCEPT_GREEDY)
+    path, alen, bonus = run_accept_gpu(target, None, tb, B.ACCEPT_GREEDY, max_path=16)
+    compare(tb, res, path, alen, bonus)
+    assert res["path"][0][:2] == [0, c]

@@ -9,7 +9,7 @@ import pytest
 import torch
 
 import oracle
-from gpu_cases import ensure_built, f32, i32
+from gpu_cases import ensure_built, f32, f32_rows, i32
 from paper_2512_21857_gb300 import binding as B
 from paper_2512_21857_gb300 import synth
 from test_parity_accept_compact import ACCEPT_MARGIN, SAMPLE_MARGIN, compare
@@ -74,8 +74,10 @@ def run_accept_cfg(tc, tu, dc, du, tb, mode, ua=None, us=None, T=1.0, max_path=1
     alen = torch.empty(Bn, dtype=torch.int32, device=dev)
     bonus = torch.empty(Bn, dtype=torch.int32, device=dev)
     opt = lambda x: None if x is None else f32(x)  # noqa: E731
-    B.adt_tree_accept_cfg(f32(tc), f32(tu), opt(dc), opt(du), i32(tb.tokens), i32(tb.parents), i32(tb.node_offsets),
-                          cfg_scale=SCALE, B=Bn, V=tc.shape[1], max_nodes=int(np.diff(tb.node_offsets).max()),
+    rows_ = lambda x: None if x is None else f32_rows(x)  # noqa: E731
+    B.adt_tree_accept_cfg(rows_(tc), rows_(tu), rows_(dc), rows_(du), i32(tb.tokens), i32(tb.parents),
+                          i32(tb.node_offsets), cfg_scale=SCALE, B=Bn, V=tc.shape[1],
+                          max_nodes=int(np.diff(tb.node_offsets).max()),
                           mode=mode, u_accept=opt(ua), u_sample=opt(us), temperature=T, path=path,
                           max_path=max_path, accept_len=alen, bonus_token=bonus)
     torch.cuda.synchronize()
@@ -98,7 +100,7 @@ def rows(tb, V, seed, plant):
     return tc, tu, dc, du
 
 
-@pytest.mark.parametrize("sizes,V", [([26], 16384), ([64, 1, 33, 7], 65536)])
+@pytest.mark.parametrize("sizes,V", [([26], 16384), ([64, 1, 33, 7], 65536), ([9, 4], 4099)])
 def test_accept_cfg_greedy_matches_oracle(sizes, V):
     seed = 900 + sum(sizes)
     tb = synth.tree_batch(sizes, V, seed)
