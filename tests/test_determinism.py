@@ -83,3 +83,36 @@ def test_7b_step_replays_are_bit_identical(plant):
         for name in outs:
             assert torch.equal(getattr(step, name), first[name]), f"replay {rep}: {name} differs"
     assert B.adt_get_device_error() == 0
+
+
+def test_ragged_batch_step_replays_are_bit_identical():
+    """The ragged eight-image batch at the 7B head shape (prefixes 640-2352,
+    per-image depth and width, each image's draft chain on its own stream,
+    one split per (tree, head) in longest-prefix-first slot order), four
+    layers: 21 graph replays give bit-identical outputs."""
+    kv = [751, 1596, 1444, 640, 1427, 1245, 2352, 1248]
+    shape = StepShape(layers=4, H=32, Hkv=32, D=128, V=65536, kv_len=kv, depth=[4, 7, 8, 7, 6, 6, 7, 6],
+                      width=[6, 8, 4, 2, 2, 1, 6, 4], max_nodes=64, mode=B.ACCEPT_GREEDY)
+    step = TreeVerifyStep(shape, keep_layer_outputs=True)
+    _fill(step, 23)
+    s = torch.cuda.Stream()
+    B.adt_get_device_error()
+    with torch.cuda.stream(s):
+        step.launch(s)
+    torch.cuda.synchronize()
+    outs = ("tokens", "parents", "attn_out", "path", "accept_len", "bonus", "kv_len_out", "k_cache", "v_cache")
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(g, stream=s):
+            step.launch(s)
+        g.replay()
+    torch.cuda.synchronize()
+    assert B.adt_get_device_error() == 0
+    first = {name: getattr(step, name).clone() for name in outs}
+    for rep in range(20):
+        with torch.cuda.stream(s):
+            g.replay()
+        torch.cuda.synchronize()
+        for name in outs:
+            assert torch.equal(getattr(step, name), first[name]), f"replay {rep}: {name} differs"
+    assert B.adt_get_device_error() == 0
