@@ -458,7 +458,7 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
             }
         }
       }
-      for (int i = 4 * c4 + tid; i < cnt; i += kThreads) {  // the slice's last (V % 4) values
+      for (int i = 4 * c4 + tid; i < cnt; i += kThreads) {  // the last slice's final cnt % 4 values
         float x = __ldg(trow + lo + i);
         if (trow_u) x = adt::cfg_combine(x, __ldg(trow_u + lo + i), p.cfg);
         if (better(x, lo + i, bv, bi)) {
