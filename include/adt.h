@@ -214,6 +214,9 @@ adt_status adt_tree_attn_noalloc(const adt_bf16* q, const adt_bf16* k_cache,
  * child_token, child_parent [device] int32 [F*k_child];
  * child_logp (or NULL), child_score [device] fp32 [F*k_child];
  * keep_idx [device] int32 [k_keep]; next_score, next_id [device] or NULL.
+ * keep_idx may be NULL (then next_score and next_id must be NULL too) when
+ * no next frontier is wanted, e.g. for the tree's last layer: the children
+ * are written as above and the selection across rows is skipped.
  * Logits must be finite (NaN is outside the domain and not checked).
  * ------------------------------------------------------------------------ */
 size_t adt_tree_expand_workspace_size(int32_t F, int32_t V, int32_t k_child);

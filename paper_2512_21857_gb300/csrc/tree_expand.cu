@@ -438,7 +438,9 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
     if (p.clogp) p.clogp[c] = static_cast<float>(lp);
     p.cscore[c] = score;
     p.cpar[c] = f_id;
-    if (p.F == 1) {
+    if (!p.keep) {
+      // No next frontier wanted (the tree's last layer).
+    } else if (p.F == 1) {
       // One row: its children are already in score order (the score grows
       // with the log-probability; ties keep the lower index, as the
       // cross-row ranking would), so the next frontier is their first k_keep.
@@ -451,7 +453,7 @@ __global__ void __launch_bounds__(kThreads) expand_kernel(const ExpandParams p) 
       p.cross_keys[c] = adt::select_key(score, static_cast<uint32_t>(c));
     }
   }
-  if (p.F == 1) return;
+  if (p.F == 1 || !p.keep) return;
   // The row's cross keys are written (CTA order); the ticket's release
   // publishes them at device scope and its acquire, in the last row, makes
   // every row's keys visible.
@@ -772,7 +774,8 @@ static adt_status expand_impl(const float* logits, const float* logits_u, float 
                               int32_t* child_token, float* child_logp, float* child_score,
                               int32_t* child_parent, int32_t* keep_idx, float* next_score, int32_t* next_id,
                               void* workspace, size_t workspace_bytes, void* stream) {
-  ADT_REQUIRE(logits && frontier_score && child_token && child_score && child_parent && keep_idx);
+  ADT_REQUIRE(logits && frontier_score && child_token && child_score && child_parent);
+  ADT_REQUIRE(keep_idx || (!next_score && !next_id));
   if (logits_u) ADT_REQUIRE(adt::aligned16(logits_u) && cfg_scale > -1e30f && cfg_scale < 1e30f);
   ADT_REQUIRE(F >= 1 && F <= kMaxRows && V >= 1 && V <= (1 << 24));
   ADT_REQUIRE(k_child >= 1 && k_child <= kMaxK && k_child <= V);

@@ -330,11 +330,13 @@ class Decoder:
             keep = torch.empty(width, dtype=torch.int32, device=dev)
             nsc = torch.empty(width, dtype=torch.float32, device=dev)
             nid = torch.empty(width, dtype=torch.int32, device=dev)
+            last = d + 1 == depth  # no next frontier after the last layer
             B.adt_tree_expand(logits, fscore, fid, F=F, V=s.vocab, k_child=width, k_keep=width, child_id_base=base,
                               child_token=pool_tok[base:base + F * width], child_logp=pool_lp[base:base + F * width],
                               child_score=pool_sc[base:base + F * width],
-                              child_parent=pool_par[base:base + F * width], keep_idx=keep, next_score=nsc,
-                              next_id=nid, workspace=self.ws_expand)
+                              child_parent=pool_par[base:base + F * width], keep_idx=None if last else keep,
+                              next_score=None if last else nsc, next_id=None if last else nid,
+                              workspace=self.ws_expand)
             if d + 1 < depth:
                 # the kept candidates join the draft tree (their parents: frontier nodes)
                 kept = nid.long()

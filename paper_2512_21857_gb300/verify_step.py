@@ -151,14 +151,17 @@ class TreeVerifyStep:
         for d in range(s.depth[b]):
             F = 1 if d == 0 else k
             nxt = d % 2
+            last = d == s.depth[b] - 1  # the tree's last layer: no next frontier
             B.adt_tree_expand(rows[d, :F], fscore, fid, F=F, V=s.V, k_child=k, k_keep=k,
                               temperature=1.0, child_id_base=base,
                               child_token=self.pool_tok[b][base:base + F * k],
                               child_logp=self.pool_logp[b][base:base + F * k],
                               child_score=self.pool_score[b][base:base + F * k],
                               child_parent=self.pool_par[b][base:base + F * k],
-                              keep_idx=keep[:k], next_score=front_score[nxt, :k],
-                              next_id=front_id[nxt, :k], workspace=self.ws_expand[b], stream=stream)
+                              keep_idx=None if last else keep[:k],
+                              next_score=None if last else front_score[nxt, :k],
+                              next_id=None if last else front_id[nxt, :k], workspace=self.ws_expand[b],
+                              stream=stream)
             fscore, fid = front_score[nxt, :k], front_id[nxt, :k]
             base += F * k
         if not rerank:

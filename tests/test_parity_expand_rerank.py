@@ -260,3 +260,31 @@ def test_expand_many_values_at_the_bound(n_top):
     ref = oracle.tree_expand(logits, fscore, k, 8)
     assert got["child_token"][:k].tolist() == pos[:k].tolist()
     check_expand(got, ref, 8)
+
+
+def test_expand_without_next_frontier():
+    """keep_idx, next_score and next_id NULL (a tree's last layer): the
+    children are the oracle's, and the shared workspace's counter stays at
+    zero for the next call, which selects a frontier as usual."""
+    F, V, k = 8, 65536, 8
+    logits = synth.f32_normal((F, V), 77, "logits", std=3.0)
+    fscore = synth.f32_normal((F,), 77, "fs", std=1.0) - 2.0
+    ref = oracle.tree_expand(logits, fscore, k, k)
+    dev = "cuda"
+    ws = B.zeroed_workspace(B.adt_tree_expand_workspace_size(F, V, k))
+    out = dict(child_token=torch.empty(F * k, dtype=torch.int32, device=dev),
+               child_logp=torch.empty(F * k, dtype=torch.float32, device=dev),
+               child_score=torch.empty(F * k, dtype=torch.float32, device=dev),
+               child_parent=torch.empty(F * k, dtype=torch.int32, device=dev))
+    B.adt_tree_expand(f32(logits), f32(fscore), None, F=F, V=V, k_child=k, k_keep=k, keep_idx=None,
+                      workspace=ws, **out)
+    torch.cuda.synchronize()
+    assert np.array_equal(out["child_token"].cpu().numpy(), ref["child_token"])
+    assert np.array_equal(out["child_parent"].cpu().numpy(), ref["child_parent"])
+    assert np.abs(out["child_score"].cpu().numpy() - ref["child_score"]).max() <= TOL
+    assert int(ws[:16640].cpu().sum()) == 0
+    got, _ = run_expand(logits, fscore, None, k, k, ws=ws)
+    check_expand(got, ref, k)
+    with pytest.raises(B.AdtError):
+        B.adt_tree_expand(f32(logits), f32(fscore), None, F=F, V=V, k_child=k, k_keep=k, keep_idx=None,
+                          next_score=torch.empty(k, dtype=torch.float32, device=dev), workspace=ws, **out)
