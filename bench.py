@@ -811,8 +811,8 @@ def main():
                 "d2h_bytes_per_step": r["d2h"]},
         "expansion": {"kernel": "expand_kernel", "calls_per_step": r["expand_calls"],
                       "avg_call_us": r["expand_us"],
-                      "note": "image 0's draft-tree expansion calls (F = 1, then the width) replayed alone "
-                              "back to back in a graph"},
+                      "note": "image 0's draft-tree expansion calls (F = 1, then the width; the last one "
+                              "without a next frontier) replayed alone back to back in a graph"},
         "gpu_launches": r["launches"],
         "clocks": r["clocks"],
         "cpu_baseline": cpu,
