@@ -76,12 +76,6 @@ __device__ __forceinline__ df df_mul_f(df x, float f) {
 
 __device__ __forceinline__ double to_double(df x) { return static_cast<double>(x.hi) + static_cast<double>(x.lo); }
 
-// The double-float nearest to an fp64 value (hi = its fp32 rounding).
-__device__ __forceinline__ df from_double(double v) {
-  const float hi = __double2float_rn(v);
-  return df{hi, __double2float_rn(v - static_cast<double>(hi))};
-}
-
 // 2^(j/64), j = 0 .. 63, as double-floats (hi, lo), evaluated in exact
 // decimal arithmetic: the table of the reduction in df_exp_diff.  A kernel
 // copies it to shared memory (exp_table_to_smem) and passes that copy.
@@ -160,6 +154,21 @@ __device__ __forceinline__ df df_exp_diff(float a, float b, const float2* tab) {
 // max(0, x) for a normalised double-float (its sign is hi's sign).
 __device__ __forceinline__ df df_max0(df x) { return x.hi > 0.f ? x : df{0.f, 0.f}; }
 
+// x < y for normalised double-floats: the sign of their difference.
+__device__ __forceinline__ bool df_less(df x, df y) { return df_add(x, df_neg(y)).hi < 0.f; }
+
+// 1 / y for a normalised double-float y != 0: one Newton-Raphson step from
+// the correctly rounded fp32 reciprocal t of y.hi, r = t + t (1 - y t), with
+// 1 - y t formed from the exact product y.hi t (two_prod) less y.lo t.  The
+// residual 1 - y t is about 2^-24, so the step leaves a relative error near
+// 2^-46.
+__device__ __forceinline__ df df_recip(df y) {
+  const float t = __frcp_rn(y.hi);
+  const df p = two_prod(y.hi, t);
+  const float e = __fsub_rn(__fsub_rn(__fsub_rn(1.f, p.hi), p.lo), __fmul_rn(y.lo, t));
+  return fast_two_sum(t, __fmul_rn(t, e));
+}
+
 // Running sum of many double-float terms: the leading words summed with
 // TwoSum, their errors and the trailing words gathered in a second word
 // (a compensated sum; its error stays near n u^2 of the sum for the n
@@ -171,7 +180,6 @@ struct Acc {
     s = t.hi;
     c = __fadd_rn(c, __fadd_rn(t.lo, x.lo));
   }
-  __device__ __forceinline__ double value() const { return static_cast<double>(s) + static_cast<double>(c); }
   __device__ __forceinline__ df value_df() const { return fast_two_sum(s, c); }
 };
 

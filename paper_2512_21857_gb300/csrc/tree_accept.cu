@@ -23,7 +23,6 @@ namespace {
 
 constexpr int kThreads = 512;
 constexpr int kMaxNodes = 1024;
-constexpr int kMaxCluster = 16;
 
 struct AcceptParams {
   const float* target;
@@ -54,7 +53,7 @@ struct AcceptParams {
 // Values a CTA publishes to its cluster; two copies alternate so that one
 // barrier per exchange suffices.
 struct Slot {
-  double d[2];
+  float2 g[2];  // double-float values (hi, lo)
   float f[2];
   int i[2];
 };
@@ -70,9 +69,9 @@ struct Shared {
   int ired[32];
   float2 exptab[64];  // 2^(j/64) as double-floats (the double-float exponential's table)
   float2 dfred[32];   // double-float block reductions
-  // Scalars thread 0 derives from the cluster's published values (in fp64,
-  // once per CTA: FP64 runs at a small fraction of the FP32 rate, so every
-  // thread repeating them would cost microseconds) and hands to the block.
+  float2 dfpre[32];   // exclusive prefix of the warps' double-float totals
+  // Scalars thread 0 derives from the cluster's published values (in
+  // double-float, once per CTA) and hands to the block.
   float2 bf[4];
   int bi[4];
   int nkids;
@@ -98,6 +97,23 @@ __device__ __forceinline__ bool better(float v, int i, float bv, int bi) {
   return v > bv || (v == bv && i < bi);
 }
 
+// The cluster's published double-float values g[k] summed over its CTAs:
+// lane c (< csize) of the calling warp reads CTA c's slot, so the reads go
+// out together instead of one after another, and the lanes combine them by
+// shuffles.  Every CTA runs the same operations on the same values, so all
+// get the same sum; lane 0's is the one used.
+__device__ __forceinline__ dfl::df warp_cluster_sum(Walker& w, int k) {
+  const int lane = threadIdx.x & 31;
+  dfl::df v{0.f, 0.f};
+  if (lane < w.csize) {
+    const float2 g = w.peer(lane)->g[k];
+    v = dfl::df{g.x, g.y};
+  }
+  for (int o = 16; o > 0; o >>= 1)
+    v = dfl::df_add(v, dfl::df{__shfl_xor_sync(adt::kFullMask, v.hi, o), __shfl_xor_sync(adt::kFullMask, v.lo, o)});
+  return v;
+}
+
 // The sampling modes' slices of p and q.  Slice<true>: double-float
 // entries (hi, lo), exponentials and every update in double-float, so the
 // decisions the walk takes from them (u q(x) < p(x), the inverse-CDF draw)
@@ -113,7 +129,6 @@ struct Slice<false> {
   static __device__ __forceinline__ E logit(float x) { return x; }
   static __device__ __forceinline__ float value_hi(E v) { return v; }
   static __device__ __forceinline__ E exp_diff(float x, float M, const float2*) { return expf(x - M); }
-  static __device__ __forceinline__ double d(E v) { return v; }
   static __device__ __forceinline__ bool pos(E v) { return v > 0.f; }
   static __device__ __forceinline__ E zero() { return 0.f; }
   static __device__ __forceinline__ dfl::df as_df(E v) { return dfl::df{v, 0.f}; }
@@ -124,7 +139,6 @@ struct Slice<false> {
   struct Acc {
     float a = 0.f;
     __device__ __forceinline__ void add(E v) { a += v; }
-    __device__ __forceinline__ double value() const { return a; }
     __device__ __forceinline__ dfl::df value_df() const { return dfl::df{a, 0.f}; }
   };
 };
@@ -138,7 +152,6 @@ struct Slice<true> {
     const dfl::df e = dfl::df_exp_diff(x, M, tab);
     return make_float2(e.hi, e.lo);
   }
-  static __device__ __forceinline__ double d(E v) { return static_cast<double>(v.x) + static_cast<double>(v.y); }
   static __device__ __forceinline__ bool pos(E v) { return v.x > 0.f; }
   static __device__ __forceinline__ E zero() { return make_float2(0.f, 0.f); }
   static __device__ __forceinline__ dfl::df as_df(E v) { return dfl::df{v.x, v.y}; }
@@ -155,7 +168,6 @@ struct Slice<true> {
   struct Acc {
     dfl::Acc a;
     __device__ __forceinline__ void add(E v) { a.add(dfl::df{v.x, v.y}); }
-    __device__ __forceinline__ double value() const { return a.value(); }
     __device__ __forceinline__ dfl::df value_df() const { return a.value_df(); }
   };
 };
@@ -261,42 +273,58 @@ __device__ float slice_max(const typename Slice<kDF>::E* buf, int Vs, Shared* sh
 // in the cluster's slices: smallest t with sum_{j<=t} w_j > u * sum_j w_j.
 // Returns the token id on every CTA.
 template <bool kDF>
-__device__ int cluster_sample(Walker& w, const typename Slice<kDF>::E* buf, int lo, int cnt, double u, Shared* sh) {
+__device__ int cluster_sample(Walker& w, const typename Slice<kDF>::E* buf, int lo, int cnt, float u, Shared* sh) {
   // 1. per-CTA slice totals (each thread owns a contiguous run), published.
+  // A thread reads its run starting at offset tid mod len, wrapping around:
+  // at the same step the threads of a half-warp then touch different banks
+  // (in index order every thread would hit the same bank).
   const int per = (cnt + kThreads - 1) / kThreads;
   const int b0 = min(cnt, static_cast<int>(threadIdx.x) * per), b1 = min(cnt, b0 + per);
   typename Slice<kDF>::Acc racc;
   int last_pos = -1;
-  for (int i = b0; i < b1; ++i) {
-    racc.add(buf[i]);
-    if (Slice<kDF>::pos(buf[i])) last_pos = i;
+  {
+    const int len = b1 - b0;
+    int j = len > 0 ? static_cast<int>(threadIdx.x) % len : 0;
+    for (int k = 0; k < len; ++k) {
+      const int i = b0 + j;
+      racc.add(buf[i]);
+      if (Slice<kDF>::pos(buf[i])) last_pos = max(last_pos, i);
+      if (++j == len) j = 0;
+    }
   }
   const dfl::df run = racc.value_df();
   const dfl::df tot = block_sum_df(run, sh);
-  if (threadIdx.x == 0) w.publish_slot()->d[0] = dfl::to_double(tot);
+  if (threadIdx.x == 0) w.publish_slot()->g[0] = make_float2(tot.hi, tot.lo);
   w.exchange();
-  if (threadIdx.x == 0) {
-    double grand = 0.0, base = 0.0;
-    for (int c = 0; c < w.csize; ++c) {
-      const double t = w.peer(c)->d[0];
-      if (c < w.rank) base += t;
-      grand += t;
+  if (threadIdx.x < 32) {
+    // Lane c reads CTA c's total; an inclusive scan over the lanes gives
+    // every CTA's cumulative total (the grand total in lane csize - 1).
+    const int lane = threadIdx.x;
+    dfl::df t{0.f, 0.f};
+    if (lane < w.csize) {
+      const float2 g = w.peer(lane)->g[0];
+      t = dfl::df{g.x, g.y};
     }
-    const double target = u * grand;
+    dfl::df incl = t;
+    for (int o = 1; o < 32; o <<= 1) {
+      const dfl::df y{__shfl_up_sync(adt::kFullMask, incl.hi, o), __shfl_up_sync(adt::kFullMask, incl.lo, o)};
+      if (lane >= o) incl = dfl::df_add(incl, y);
+    }
+    const dfl::df grand{__shfl_sync(adt::kFullMask, incl.hi, w.csize - 1),
+                        __shfl_sync(adt::kFullMask, incl.lo, w.csize - 1)};
+    const int br = w.rank > 0 ? w.rank - 1 : 0;
+    const dfl::df before{__shfl_sync(adt::kFullMask, incl.hi, br), __shfl_sync(adt::kFullMask, incl.lo, br)};
+    const dfl::df base = w.rank > 0 ? before : dfl::df{0.f, 0.f};
+    const dfl::df target = dfl::df_mul_f(grand, u);
     // Owner: first CTA whose cumulative total passes the target; else the
     // last CTA with mass.
-    int owner = -1, last_nz = -1;
-    double acc = 0.0;
-    for (int c = 0; c < w.csize; ++c) {
-      const double t = w.peer(c)->d[0];
-      if (owner < 0 && acc + t > target) owner = c;
-      if (t > 0.0) last_nz = c;
-      acc += t;
+    const unsigned pass = __ballot_sync(adt::kFullMask, lane < w.csize && dfl::df_less(target, incl));
+    const unsigned mass = __ballot_sync(adt::kFullMask, lane < w.csize && t.hi > 0.f);
+    if (lane == 0) {
+      sh->bi[0] = pass ? __ffs(pass) - 1 : (mass ? 31 - __clz(mass) : 0);
+      sh->bf[0] = make_float2(base.hi, base.lo);
+      sh->bf[1] = make_float2(-target.hi, -target.lo);
     }
-    sh->bi[0] = owner < 0 ? (last_nz < 0 ? 0 : last_nz) : owner;
-    const dfl::df bdf = dfl::from_double(base), tdf = dfl::from_double(-target);
-    sh->bf[0] = make_float2(bdf.hi, bdf.lo);
-    sh->bf[1] = make_float2(tdf.hi, tdf.lo);
   }
   __syncthreads();
   const int owner = sh->bi[0];
@@ -318,17 +346,30 @@ __device__ int cluster_sample(Walker& w, const typename Slice<kDF>::E* buf, int 
       sh->last_pos = -1;
     }
     __syncthreads();
-    dfl::df acc = base;
-    for (int j = 0; j < warp; ++j) acc = dfl::df_add(acc, dfl::df{sh->dfred[j].x, sh->dfred[j].y});
+    if (warp == 0) {
+      // exclusive prefix of the warps' totals, one scan in warp 0
+      dfl::df wt = lane < kThreads / 32 ? dfl::df{sh->dfred[lane].x, sh->dfred[lane].y} : dfl::df{0.f, 0.f};
+      for (int o = 1; o < 32; o <<= 1) {
+        const dfl::df y{__shfl_up_sync(adt::kFullMask, wt.hi, o), __shfl_up_sync(adt::kFullMask, wt.lo, o)};
+        if (lane >= o) wt = dfl::df_add(wt, y);
+      }
+      const dfl::df prev{__shfl_up_sync(adt::kFullMask, wt.hi, 1), __shfl_up_sync(adt::kFullMask, wt.lo, 1)};
+      if (lane < kThreads / 32) sh->dfpre[lane] = lane == 0 ? make_float2(0.f, 0.f) : make_float2(prev.hi, prev.lo);
+    }
+    __syncthreads();
     // The running CDF in double-float, compared with the target through the
-    // sign of their difference.
+    // sign of their difference.  A run whose end does not pass the target
+    // cannot hold the draw and is not walked.
+    dfl::df acc = dfl::df_add(base, dfl::df{sh->dfpre[warp].x, sh->dfpre[warp].y});
     acc = dfl::df_add(acc, dfl::df_add(incl, dfl::df_neg(run)));
     if (last_pos >= 0) atomicMax(&sh->last_pos, last_pos);
-    for (int i = b0; i < b1; ++i) {
-      acc = dfl::df_add(acc, Slice<kDF>::as_df(buf[i]));
-      if (Slice<kDF>::pos(buf[i]) && dfl::df_add(acc, ntgt).hi > 0.f) {
-        atomicMin(&sh->found, i);
-        break;
+    if (dfl::df_add(dfl::df_add(acc, run), ntgt).hi > 0.f) {
+      for (int i = b0; i < b1; ++i) {
+        acc = dfl::df_add(acc, Slice<kDF>::as_df(buf[i]));
+        if (Slice<kDF>::pos(buf[i]) && dfl::df_add(acc, ntgt).hi > 0.f) {
+          atomicMin(&sh->found, i);
+          break;
+        }
       }
     }
     __syncthreads();
@@ -472,13 +513,20 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
         w.publish_slot()->i[0] = bi;
       }
       w.exchange();
+      // lane c reads CTA c's candidate; the warp's argmax over the lanes
       float gvv = -INFINITY;
       int g = 0x7fffffff;
-      for (int c = 0; c < w.csize; ++c) {
-        const Slot* s = w.peer(c);
-        if (better(s->f[0], s->i[0], gvv, g)) {
-          gvv = s->f[0];
-          g = s->i[0];
+      if ((tid & 31) < w.csize) {
+        const Slot* s = w.peer(tid & 31);
+        gvv = s->f[0];
+        g = s->i[0];
+      }
+      for (int o = 16; o > 0; o >>= 1) {
+        const float ov = __shfl_xor_sync(adt::kFullMask, gvv, o);
+        const int oi = __shfl_xor_sync(adt::kFullMask, g, o);
+        if (better(ov, oi, gvv, g)) {
+          gvv = ov;
+          g = oi;
         }
       }
       w.flip();
@@ -522,27 +570,29 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
     }
     w.exchange();
     float Mp = -INFINITY, Mq = -INFINITY;
-    for (int c = 0; c < w.csize; ++c) {
-      Mp = fmaxf(Mp, w.peer(c)->f[0]);
-      Mq = fmaxf(Mq, w.peer(c)->f[1]);
+    if ((tid & 31) < w.csize) {  // lane c reads CTA c's maxima
+      Mp = w.peer(tid & 31)->f[0];
+      Mq = w.peer(tid & 31)->f[1];
     }
+    Mp = adt::warp_max(Mp);
+    Mq = adt::warp_max(Mq);
     w.flip();
     const dfl::df sp_loc = exp_in_place<kDF>(pbuf, p.Vs, Mp, &sh);
     const dfl::df sq_loc = need_q ? exp_in_place<kDF>(qbuf, p.Vs, Mq, &sh) : dfl::df{0.f, 0.f};
     if (tid == 0) {
-      w.publish_slot()->d[0] = dfl::to_double(sp_loc);
-      w.publish_slot()->d[1] = dfl::to_double(sq_loc);
+      w.publish_slot()->g[0] = make_float2(sp_loc.hi, sp_loc.lo);
+      w.publish_slot()->g[1] = make_float2(sq_loc.hi, sq_loc.lo);
     }
     w.exchange();
     // The row totals, formed once (thread 0 keeps them for the decisions) and
     // handed to the block as double-float reciprocals.
-    double Sp = 0.0, Sq = 0.0;
+    dfl::df Sp{0.f, 0.f}, Sq{0.f, 0.f};
+    if (tid < 32) {
+      Sp = warp_cluster_sum(w, 0);
+      Sq = warp_cluster_sum(w, 1);
+    }
     if (tid == 0) {
-      for (int c = 0; c < w.csize; ++c) {
-        Sp += w.peer(c)->d[0];
-        Sq += w.peer(c)->d[1];
-      }
-      const dfl::df ip = dfl::from_double(1.0 / Sp), iq = dfl::from_double(Sq > 0.0 ? 1.0 / Sq : 0.0);
+      const dfl::df ip = dfl::df_recip(Sp), iq = Sq.hi > 0.f ? dfl::df_recip(Sq) : dfl::df{0.f, 0.f};
       sh.bf[0] = make_float2(ip.hi, ip.lo);
       sh.bf[1] = make_float2(iq.hi, iq.lo);
     }
@@ -560,9 +610,10 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
     }
 
     // The children in ascending index.  Thread 0 reads p(x), q(x) from the
-    // owning CTA, takes the decision in fp64 and hands it to the block.
+    // owning CTA, takes the decision in double-float and hands it to the
+    // block.
     int nxt = -1;
-    double e_rej = 0.0;  // SPEC_DET, thread 0: rejected unnormalised mass
+    dfl::df e_rej{0.f, 0.f};  // SPEC_DET, thread 0: rejected unnormalised mass
     int nrej = 0;        // SPEC_DET: rejected tokens (in sh.rejected)
     for (int j = 0; j < nk; ++j) {
       const int c = sh.kids[j];
@@ -573,24 +624,24 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
       }
       const int owner = x / p.Vs, off = x - owner * p.Vs;
       if (tid == 0) {
-        const double u = static_cast<double>(p.ua[node0 + c]);
+        // u < p(x) / denom is taken as u denom < p(x): no division.
+        const float u = p.ua[node0 + c];
         if (!spec) {
           bool dup = false;
           for (int r = 0; r < nrej; ++r) dup |= sh.rejected[r] == x;
-          const double ex = dup ? 0.0 : SL::d(*cl.map_shared_rank(pbuf + off, owner));
-          const double denom = Sp - e_rej;
-          const double px = denom > 0.0 ? ex / denom : 0.0;
-          const bool a = u < px;
+          const dfl::df ex = dup ? dfl::df{0.f, 0.f} : SL::as_df(*cl.map_shared_rank(pbuf + off, owner));
+          const dfl::df denom = dfl::df_add(Sp, dfl::df_neg(e_rej));
+          const bool a = denom.hi > 0.f && dfl::df_less(dfl::df_mul_f(denom, u), ex);
           sh.bi[1] = a;
           sh.bi[2] = !a && !dup;  // a new rejected token
           if (!a && !dup) {
-            e_rej += ex;
+            e_rej = dfl::df_add(e_rej, ex);
             sh.rejected[nrej] = x;
           }
         } else {
-          const double px = SL::d(*cl.map_shared_rank(pbuf + off, owner));
-          const double qx = SL::d(*cl.map_shared_rank(qbuf + off, owner));
-          sh.bi[1] = u * qx < px;
+          const dfl::df px = SL::as_df(*cl.map_shared_rank(pbuf + off, owner));
+          const dfl::df qx = SL::as_df(*cl.map_shared_rank(qbuf + off, owner));
+          sh.bi[1] = dfl::df_less(dfl::df_mul_f(qx, u), px);
           sh.bi[2] = 0;
         }
       }
@@ -608,21 +659,21 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
         const dfl::df zb = block_sum_df(zl.value_df(), &sh);
         const dfl::df qb = block_sum_df(ql.value_df(), &sh);
         if (tid == 0) {
-          w.publish_slot()->d[0] = dfl::to_double(zb);
-          w.publish_slot()->d[1] = dfl::to_double(qb);
+          w.publish_slot()->g[0] = make_float2(zb.hi, zb.lo);
+          w.publish_slot()->g[1] = make_float2(qb.hi, qb.lo);
         }
         w.exchange();  // also: every peer has finished reading px, qx
+        dfl::df Z{0.f, 0.f}, Qs{0.f, 0.f};
+        if (tid < 32) {
+          Z = warp_cluster_sum(w, 0);
+          Qs = warp_cluster_sum(w, 1);
+        }
         if (tid == 0) {
-          double Z = 0.0, Qs = 0.0;
-          for (int cc = 0; cc < w.csize; ++cc) {
-            Z += w.peer(cc)->d[0];
-            Qs += w.peer(cc)->d[1];
-          }
-          const dfl::df iz = dfl::from_double(Z > 0.0 ? 1.0 / Z : 0.0);
-          const dfl::df iqs = dfl::from_double(Qs > 0.0 ? 1.0 / Qs : 0.0);
+          const dfl::df iz = Z.hi > 0.f ? dfl::df_recip(Z) : dfl::df{0.f, 0.f};
+          const dfl::df iqs = Qs.hi > 0.f ? dfl::df_recip(Qs) : dfl::df{0.f, 0.f};
           sh.bf[0] = make_float2(iz.hi, iz.lo);
           sh.bf[1] = make_float2(iqs.hi, iqs.lo);
-          sh.bi[0] = Z > 0.0;
+          sh.bi[0] = Z.hi > 0.f;
         }
         __syncthreads();
         w.flip();
@@ -656,7 +707,7 @@ __global__ void __launch_bounds__(kThreads) accept_kernel(const AcceptParams p) 
       }
     }
     __syncthreads();
-    bonus = cluster_sample<kDF>(w, pbuf, lo, cnt, static_cast<double>(p.us[gv]), &sh);
+    bonus = cluster_sample<kDF>(w, pbuf, lo, cnt, p.us[gv], &sh);
     break;
   }
 
